@@ -1,0 +1,161 @@
+"""CPU fp64 oracle for the per-head-window KV path -- TEST INFRASTRUCTURE.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg
+may import this package. It shares no code with the CUDA library; its only
+shared dependency is the seeded input generator (``hwkv_gen``).
+Each function states the passage of the HeadWiseKV paper it follows; the C
+source ``hwkv_oracle.c`` holds the arithmetic.
+"""
+import ctypes
+
+import numpy as np
+
+from . import build as _build
+from hwkv_gen import GenDesc
+
+FULL = 0
+_lib = None
+
+_i64p = ctypes.POINTER(ctypes.c_int64)
+_f64p = ctypes.POINTER(ctypes.c_double)
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _build.build()
+        L = ctypes.CDLL(_build.LIB)
+        L.oracle_threads.restype = ctypes.c_int
+        L.oracle_set_threads.argtypes = [ctypes.c_int]
+        L.oracle_window_lo.argtypes = [ctypes.c_int64, ctypes.c_int64]
+        L.oracle_window_lo.restype = ctypes.c_int64
+        L.oracle_attend.argtypes = [ctypes.c_void_p] * 3 + [ctypes.c_int64, ctypes.c_int64,
+                                                            ctypes.c_double, ctypes.c_void_p,
+                                                            ctypes.c_void_p]
+        L.oracle_attend.restype = ctypes.c_double
+        L.oracle_window_attention_bf16.argtypes = [
+            ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p,
+            ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+            ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p]
+        L.oracle_window_attention_bf16.restype = ctypes.c_int
+        L.oracle_window_attention_gen.argtypes = [
+            ctypes.POINTER(GenDesc), ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int64,
+            ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p]
+        L.oracle_window_attention_gen.restype = ctypes.c_int
+        L.oracle_ring_positions.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p]
+        L.oracle_ring_positions.restype = ctypes.c_int
+        L.oracle_ring_expected_gen.argtypes = [
+            ctypes.POINTER(GenDesc), ctypes.c_uint32, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p]
+        L.oracle_ring_expected_gen.restype = ctypes.c_int
+        L.oracle_retained_tokens.argtypes = [ctypes.c_int64, ctypes.c_int64]
+        L.oracle_retained_tokens.restype = ctypes.c_int64
+        L.oracle_nominal_storage.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64,
+                                             ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                             ctypes.c_int64, ctypes.c_int64]
+        L.oracle_nominal_storage.restype = ctypes.c_uint64
+        L.oracle_normalized_rate.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64,
+                                             ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                             ctypes.c_int64]
+        L.oracle_normalized_rate.restype = ctypes.c_double
+        _lib = L
+    return _lib
+
+
+def _p(a):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def threads():
+    return int(lib().oracle_threads())
+
+
+def set_threads(n):
+    lib().oracle_set_threads(int(n))
+
+
+def window_lo(p, W):
+    """Lower end of J_p(W) (Sec. 3.2), 0-based; W = 0 is full history."""
+    return int(lib().oracle_window_lo(p, W))
+
+
+def attend(q, K, V, gamma):
+    """Eq. conditional-attention-weight / conditional-attention over an explicit set.
+
+    q [d], K [n, d], V [n, d] float64. Returns (o [d], pi [n])."""
+    q = np.ascontiguousarray(q, dtype=np.float64)
+    K = np.ascontiguousarray(K, dtype=np.float64)
+    V = np.ascontiguousarray(V, dtype=np.float64)
+    n, d = K.shape
+    o = np.zeros(d)
+    pi = np.zeros(max(n, 1))
+    lib().oracle_attend(_p(q), _p(K), _p(V), n, d, float(gamma), _p(o), _p(pi))
+    return o, pi[:n]
+
+
+def window_attention_bf16(Q, pos, Kp, Vp, W, gamma):
+    """Window-limited attention of rows Q [R, d] (bf16 bits) at positions pos [R]
+    over K/V histories Kp, Vp [T, d] (bf16 bits, row = absolute position).
+    Returns (O [R, d] float64, sum_pi [R])."""
+    Q = np.ascontiguousarray(Q, dtype=np.uint16)
+    Kp = np.ascontiguousarray(Kp, dtype=np.uint16)
+    Vp = np.ascontiguousarray(Vp, dtype=np.uint16)
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    R, d = Q.shape
+    T = Kp.shape[0]
+    O = np.zeros((R, d))
+    sp = np.zeros(R)
+    rc = lib().oracle_window_attention_bf16(_p(Q), d, _p(pos), R, _p(Kp), _p(Vp), d, T, d,
+                                            int(W), float(gamma), _p(O), _p(sp))
+    if rc != 0:
+        raise ValueError("oracle_window_attention_bf16: bad arguments (rc=%d)" % rc)
+    return O, sp
+
+
+def window_attention_gen(g, layer, b, kvh, qheads, pos, d, W, gamma):
+    """Same definition with q/K/V regenerated from the seeded generator.
+    Row r: query head qheads[r] of batch row b at position pos[r], reading KV head kvh."""
+    qh = np.ascontiguousarray(qheads, dtype=np.int32)
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    R = len(pos)
+    O = np.zeros((R, d))
+    sp = np.zeros(R)
+    rc = lib().oracle_window_attention_gen(ctypes.byref(g), layer, b, kvh, _p(qh), _p(pos), R,
+                                           d, int(W), float(gamma), _p(O), _p(sp))
+    if rc != 0:
+        raise ValueError("oracle_window_attention_gen: bad arguments (rc=%d)" % rc)
+    return O, sp
+
+
+def ring_positions(t, cap):
+    """Sec. 3.3 residency as a ring: position held by each slot (-1 = empty)."""
+    out = np.zeros(cap, dtype=np.int64)
+    if lib().oracle_ring_positions(t, cap, _p(out)) != 0:
+        raise ValueError("bad ring arguments")
+    return out
+
+
+def ring_expected_gen(g, tensor, layer, b, kvh, d, t, cap):
+    out = np.zeros((cap, d), dtype=np.uint16)
+    if lib().oracle_ring_expected_gen(ctypes.byref(g), tensor, layer, b, kvh, d, t, cap,
+                                      _p(out)) != 0:
+        raise ValueError("bad ring arguments")
+    return out
+
+
+def retained_tokens(W, C):
+    """r_C(w) (Sec. 3.1)."""
+    return int(lib().oracle_retained_tokens(W, C))
+
+
+def nominal_storage(windows, C, dK, dV, bK=2, bV=2, batch=1):
+    """N_C(a), Eq. nominal-storage, in bytes, times `batch` sequences."""
+    w = np.ascontiguousarray(windows, dtype=np.int64).ravel()
+    return int(lib().oracle_nominal_storage(_p(w), len(w), C, dK, dV, bK, bV, batch))
+
+
+def normalized_rate(windows, C, dK, dV, bK=2, bV=2):
+    """R_C(a), Eq. normalized-rate."""
+    w = np.ascontiguousarray(windows, dtype=np.int64).ravel()
+    return float(lib().oracle_normalized_rate(_p(w), len(w), C, dK, dV, bK, bV))

@@ -1,0 +1,270 @@
+/*
+ * hwkv_oracle.c -- TEST INFRASTRUCTURE. A plain, slow, fp64 CPU statement of
+ * what the per-head-window KV path computes, written from the HeadWiseKV
+ * paper. Only the test suite, the smoke check and the benchmark's CPU-baseline
+ * leg load it; the library never does, and it shares no code with the CUDA
+ * path (its only include besides libc is the seeded input generator).
+ *
+ * Everything here is the definition written out, with no blocking, splitting,
+ * fusion or reordering:
+ *   - retained window   J_t(w) = {max(1, t-w+1), ..., t}, J_t(full) = {1..t}
+ *                       (Sec. 3.2, definition above Eq. conditional-attention-weight),
+ *                       used 0-based: s in [max(0, p-W+1), p];
+ *   - attention         pi_s = exp(z_s) / sum_{j in J} exp(z_j),  z_s = gamma q.k_s,
+ *                       o = sum_{s in J} pi_s v_s
+ *                       (Sec. 3.2, Eq. conditional-attention-weight and
+ *                       Eq. conditional-attention; exp(z - M) / sum exp(z - M)
+ *                       with M = max z is the same quotient);
+ *   - retained count    r_C(w) = min(w, C), r_C(full) = C (Sec. 3.1);
+ *   - nominal storage   n = r_C(w) (d^K b^K + d^V b^V), N_C = sum over units
+ *                       (Sec. 3.1, Eq. nominal-storage);
+ *   - normalized rate   R_C = N_C(a) / N_C(all full) (Sec. 3.1, Eq. normalized-rate);
+ *   - physical residency: each head keeps only its latest r_t(w) K/V states
+ *                       (Sec. 3.3); stored as a ring with slot(p) = p mod cap.
+ *
+ * Windows are int64: 0 (HWKV_WINDOW_FULL) means full history; any W >= the
+ * context is equivalent to full (Sec. 3.1). bf16 inputs are widened exactly to
+ * double. Row loops may run under OpenMP; each row is computed independently.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#include "../hwkv_gen/hwkv_gen.h"
+
+#define ORACLE_FULL 0
+
+int oracle_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
+
+void oracle_set_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+#else
+  (void)n;
+#endif
+}
+
+/* exact bf16 -> double */
+static double bf16_to_double(uint16_t h) {
+  union { uint32_t u; float f; } c;
+  c.u = (uint32_t)h << 16;
+  return (double)c.f;
+}
+
+/* ---------------------------------------------------------------- windows */
+
+/* lower end of J_p(W), 0-based (Sec. 3.2); the upper end is p itself */
+int64_t oracle_window_lo(int64_t p, int64_t W) {
+  if (W == ORACLE_FULL) return 0;
+  int64_t lo = p - W + 1;
+  return lo > 0 ? lo : 0;
+}
+
+/* ------------------------------------------------------------- attention */
+
+/*
+ * Softmax attention of one query over an explicit key/value set of n rows
+ * (Eq. conditional-attention-weight, Eq. conditional-attention).
+ * q[d], K[n][d], V[n][d]; writes o[d]; returns sum of pi (1 up to rounding).
+ * pi_out, if non-NULL, receives the n weights.
+ */
+double oracle_attend(const double* q, const double* K, const double* V, int64_t n, int64_t d,
+                     double gamma, double* o, double* pi_out) {
+  double* z = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+  double M = -INFINITY;
+  for (int64_t s = 0; s < n; ++s) {
+    double dot = 0.0;
+    for (int64_t i = 0; i < d; ++i) dot += q[i] * K[s * d + i];
+    z[s] = gamma * dot;
+    if (z[s] > M) M = z[s];
+  }
+  double Z = 0.0;
+  for (int64_t s = 0; s < n; ++s) Z += exp(z[s] - M);
+  for (int64_t i = 0; i < d; ++i) o[i] = 0.0;
+  double sum_pi = 0.0;
+  for (int64_t s = 0; s < n; ++s) {
+    double pi = exp(z[s] - M) / Z;
+    sum_pi += pi;
+    if (pi_out) pi_out[s] = pi;
+    for (int64_t i = 0; i < d; ++i) o[i] += pi * V[s * d + i];
+  }
+  free(z);
+  return sum_pi;
+}
+
+/*
+ * Window-limited attention over bf16 arrays indexed by absolute position.
+ * Kp, Vp: history of one (batch row, KV head), row s at Kp + s*ld (positions
+ * 0..T-1, T > max pos). Queries: R rows, q row r at Q + r*ldq, position pos[r].
+ * Window W (0 = full). Writes O[r][d] and sum_pi[r].
+ */
+int oracle_window_attention_bf16(const uint16_t* Q, int64_t ldq, const int64_t* pos, int64_t R,
+                                 const uint16_t* Kp, const uint16_t* Vp, int64_t ld, int64_t T,
+                                 int64_t d, int64_t W, double gamma, double* O, double* sum_pi) {
+  if (R < 0 || d <= 0 || W < 0) return 1;
+  for (int64_t r = 0; r < R; ++r)
+    if (pos[r] < 0 || pos[r] >= T) return 1;
+  int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t r = 0; r < R; ++r) {
+    const int64_t p = pos[r];
+    const int64_t lo = oracle_window_lo(p, W);
+    const int64_t n = p - lo + 1;
+    double* q = (double*)malloc(sizeof(double) * (size_t)d);
+    double* K = (double*)malloc(sizeof(double) * (size_t)(n * d));
+    double* V = (double*)malloc(sizeof(double) * (size_t)(n * d));
+    if (!q || !K || !V) {
+      bad = 1;
+    } else {
+      for (int64_t i = 0; i < d; ++i) q[i] = bf16_to_double(Q[r * ldq + i]);
+      for (int64_t s = lo; s <= p; ++s)
+        for (int64_t i = 0; i < d; ++i) {
+          K[(s - lo) * d + i] = bf16_to_double(Kp[s * ld + i]);
+          V[(s - lo) * d + i] = bf16_to_double(Vp[s * ld + i]);
+        }
+      double sp = oracle_attend(q, K, V, n, d, gamma, O + r * d, NULL);
+      if (sum_pi) sum_pi[r] = sp;
+    }
+    free(q);
+    free(K);
+    free(V);
+  }
+  return bad ? 2 : 0;
+}
+
+/*
+ * The same definition, with q, K and V regenerated from the seeded generator
+ * instead of read from arrays (for contexts too large to hold on the host).
+ * Query rows: (batch row b, query head qh, position pos[r]) for r < R; the
+ * query head reads KV head kvh (its GQA group). Writes O[r][d].
+ * Two passes over J (logits, then weights and values) so no |J| x d buffer
+ * is needed.
+ */
+int oracle_window_attention_gen(const hwkv_gen_desc* g, int32_t layer, int32_t b, int32_t kvh,
+                                const int32_t* qh, const int64_t* pos, int64_t R, int32_t d,
+                                int64_t W, double gamma, double* O, double* sum_pi) {
+  if (!g || R < 0 || d <= 0 || W < 0) return 1;
+  int bad = 0;
+  const float sk = hwkv_gen_head_scale(g, HWKV_GEN_K, (uint32_t)layer, (uint32_t)kvh);
+  const float sv = hwkv_gen_head_scale(g, HWKV_GEN_V, (uint32_t)layer, (uint32_t)kvh);
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t r = 0; r < R; ++r) {
+    const int64_t p = pos[r];
+    const int64_t lo = oracle_window_lo(p, W);
+    const int64_t n = p - lo + 1;
+    double* q = (double*)malloc(sizeof(double) * (size_t)d);
+    double* kv = (double*)malloc(sizeof(double) * (size_t)d);
+    double* z = (double*)malloc(sizeof(double) * (size_t)n);
+    if (!q || !kv || !z || p < 0) {
+      bad = 1;
+    } else {
+      const float sq = hwkv_gen_head_scale(g, HWKV_GEN_Q, (uint32_t)layer, (uint32_t)qh[r]);
+      for (int32_t i = 0; i < d; ++i)
+        q[i] = bf16_to_double(hwkv_gen_elem(g, HWKV_GEN_Q, (uint32_t)layer, (uint32_t)b,
+                                            (uint32_t)qh[r], (uint64_t)p, (uint32_t)i, sq));
+      double M = -INFINITY;
+      for (int64_t s = lo; s <= p; ++s) {
+        for (int32_t i = 0; i < d; ++i)
+          kv[i] = bf16_to_double(hwkv_gen_elem(g, HWKV_GEN_K, (uint32_t)layer, (uint32_t)b,
+                                               (uint32_t)kvh, (uint64_t)s, (uint32_t)i, sk));
+        double dot = 0.0;
+        for (int32_t i = 0; i < d; ++i) dot += q[i] * kv[i];
+        z[s - lo] = gamma * dot;
+        if (z[s - lo] > M) M = z[s - lo];
+      }
+      double Z = 0.0;
+      for (int64_t s = lo; s <= p; ++s) Z += exp(z[s - lo] - M);
+      double* o = O + r * d;
+      for (int32_t i = 0; i < d; ++i) o[i] = 0.0;
+      double sp = 0.0;
+      for (int64_t s = lo; s <= p; ++s) {
+        const double pi = exp(z[s - lo] - M) / Z;
+        sp += pi;
+        for (int32_t i = 0; i < d; ++i)
+          o[i] += pi * bf16_to_double(hwkv_gen_elem(g, HWKV_GEN_V, (uint32_t)layer, (uint32_t)b,
+                                                    (uint32_t)kvh, (uint64_t)s, (uint32_t)i, sv));
+      }
+      if (sum_pi) sum_pi[r] = sp;
+    }
+    free(q);
+    free(kv);
+    free(z);
+  }
+  return bad ? 2 : 0;
+}
+
+/* ------------------------------------------------------------------ rings */
+
+/*
+ * Physical residency as a ring of capacity cap: position p lives in slot
+ * p mod cap, and after t tokens the ring holds exactly the latest min(t, cap)
+ * positions (Sec. 3.3: a head retains only its latest r_t(w) states).
+ * pos_of_slot[j] = the position held by slot j, or -1 if never written.
+ */
+int oracle_ring_positions(int64_t t, int64_t cap, int64_t* pos_of_slot) {
+  if (cap <= 0 || t < 0) return 1;
+  for (int64_t j = 0; j < cap; ++j) pos_of_slot[j] = -1;
+  const int64_t first = t > cap ? t - cap : 0;
+  for (int64_t p = first; p < t; ++p) pos_of_slot[p % cap] = p;
+  return 0;
+}
+
+/*
+ * Expected ring bytes for one (layer, batch row, KV head) after positions
+ * 0..t-1 have been fed in order: ring[j][:] = the generated K (or V) row of
+ * the position slot j holds, zero where no position is held.
+ */
+int oracle_ring_expected_gen(const hwkv_gen_desc* g, uint32_t tensor, int32_t layer, int32_t b,
+                             int32_t kvh, int32_t d, int64_t t, int64_t cap, uint16_t* ring) {
+  if (!g || cap <= 0 || t < 0 || d <= 0) return 1;
+  int64_t* pos = (int64_t*)malloc(sizeof(int64_t) * (size_t)cap);
+  if (!pos) return 2;
+  oracle_ring_positions(t, cap, pos);
+  const float s = hwkv_gen_head_scale(g, tensor, (uint32_t)layer, (uint32_t)kvh);
+  for (int64_t j = 0; j < cap; ++j)
+    for (int32_t i = 0; i < d; ++i)
+      ring[j * d + i] = pos[j] < 0 ? (uint16_t)0
+                                   : hwkv_gen_elem(g, tensor, (uint32_t)layer, (uint32_t)b,
+                                                   (uint32_t)kvh, (uint64_t)pos[j], (uint32_t)i, s);
+  free(pos);
+  return 0;
+}
+
+/* ------------------------------------------------------------- accounting */
+
+/* r_C(w) = min(w, C); r_C(full) = C  (Sec. 3.1) */
+int64_t oracle_retained_tokens(int64_t W, int64_t C) {
+  if (W == ORACLE_FULL) return C;
+  return W < C ? W : C;
+}
+
+/*
+ * N_C(a) of Eq. nominal-storage: sum over decision units of
+ * r_C(w_u) (d^K b^K + d^V b^V), in bytes, times `batch` independent sequences.
+ */
+uint64_t oracle_nominal_storage(const int64_t* W, int64_t n_units, int64_t C, int64_t dK,
+                                int64_t dV, int64_t bK, int64_t bV, int64_t batch) {
+  uint64_t total = 0;
+  for (int64_t u = 0; u < n_units; ++u)
+    total += (uint64_t)oracle_retained_tokens(W[u], C) * (uint64_t)(dK * bK + dV * bV);
+  return total * (uint64_t)batch;
+}
+
+/* R_C(a) of Eq. normalized-rate */
+double oracle_normalized_rate(const int64_t* W, int64_t n_units, int64_t C, int64_t dK,
+                              int64_t dV, int64_t bK, int64_t bV) {
+  uint64_t num = oracle_nominal_storage(W, n_units, C, dK, dV, bK, bV, 1);
+  uint64_t den = 0;
+  for (int64_t u = 0; u < n_units; ++u) den += (uint64_t)C * (uint64_t)(dK * bK + dV * bV);
+  return den ? (double)num / (double)den : 0.0;
+}
