@@ -1,0 +1,188 @@
+/*
+ * hwkv.h -- C ABI of the per-head-window KV cache library (libhwkv.so).
+ *
+ * HeadWiseKV (arXiv 2609.02029) assigns every physical KV head (layer l,
+ * head h) of each residual global-attention layer one history window a_{lh}
+ * from a codebook {w_1 < ... < w_K, full} (Sec. 3.1). At serving time each
+ * configured head reads and writes only its own K/V slice, sized to its
+ * window, instead of a mask over a full cache (Sec. 3.3; App. "Runtime
+ * Realization and Deployment", physical cache realization). This library is
+ * that runtime's hot path on one GPU: per-head ring allocation, K/V
+ * append/wrap, window-limited causal prefill attention and split-KV decode
+ * attention with a log-sum-exp merge, plus exact residency accounting.
+ *
+ * Conventions for every call
+ *  - Tensors are bf16 (2-byte) unless stated; `out` tensors are fp32.
+ *    Tensor pointers are caller-owned device memory, dense, in the stated
+ *    row-major layout, 16-byte aligned.
+ *  - Head mapping under GQA (Sec. 3.1, groups G_{lh}): query head q reads KV
+ *    head q / G with G = n_q_heads / n_kv_heads (contiguous groups).
+ *  - Positions are 0-based. A query at position p with window W attends to
+ *    key positions s in [max(0, p-W+1), p] (Sec. 3.2, the set J_t(w)); a full
+ *    head attends to [0, p]. Any W >= max_ctx is full (Sec. 3.1).
+ *  - Every call that takes `cuda_stream` (a cudaStream_t, NULL = legacy
+ *    default stream) is asynchronous and stream-ordered; argument errors are
+ *    returned before anything is launched and leave the cache unchanged.
+ *    Calls on one cache must be issued on one stream (they share the cache's
+ *    device workspace) and from one host thread at a time.
+ *  - No call throws; failures return a status and set a thread-local message
+ *    readable with hwkv_last_error().
+ */
+#ifndef HWKV_H
+#define HWKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define HWKV_API __attribute__((visibility("default")))
+#else
+#define HWKV_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  HWKV_OK = 0,
+  HWKV_EINVAL = 1,       /* bad argument or policy; nothing was launched */
+  HWKV_ENOMEM = 2,       /* arena too small or device allocation failed */
+  HWKV_ECAPACITY = 3,    /* append would exceed max_ctx on a full-history head */
+  HWKV_ECUDA = 4,        /* a CUDA runtime call or launch failed */
+  HWKV_EKERNEL = 5,      /* a kernel reported an internal error (see hwkv_sync_check) */
+  HWKV_EUNSUPPORTED = 6  /* valid request outside the built kernel set (e.g. head_dim) */
+} hwkv_status;
+
+/* windows[] entry meaning "full history" (Sec. 3.1: a_{lh} = full) */
+#define HWKV_WINDOW_FULL 0
+
+/*
+ * The policy matrix a (Sec. 3.1, Eq. for a_{lh}; App. "Runtime Realization":
+ * a static layer x KV-head matrix loaded once).
+ *   windows[l * n_kv_heads + h] = W_{lh} in tokens (> 0), or HWKV_WINDOW_FULL.
+ * A head with W >= max_ctx is stored as full. max_ctx bounds the tokens any
+ * layer will ever hold (it is the ring capacity of full heads).
+ * Supported: head_dim in {64, 128, 256}; n_q_heads / n_kv_heads <= 8;
+ * batch <= 256; n_kv_heads <= 64; the policy is copied by hwkv_alloc.
+ */
+typedef struct {
+  int32_t n_layers;
+  int32_t n_kv_heads;
+  int32_t n_q_heads;
+  int32_t head_dim;
+  int32_t batch;
+  int32_t reserved;
+  int64_t max_ctx;
+  const int64_t* windows;
+} hwkv_policy;
+
+typedef struct hwkv_cache hwkv_cache; /* opaque; owned by the library */
+
+/*
+ * Device bytes hwkv_alloc needs for `policy`: the K and V rings of every
+ * (layer, KV head, batch row) -- capacity min(W, max_ctx) tokens x head_dim
+ * bf16 each -- plus the decode workspace. Pure host computation.
+ */
+HWKV_API hwkv_status hwkv_required_bytes(const hwkv_policy* policy, size_t* arena_bytes);
+
+/*
+ * Validates `policy` (positive sizes, n_q_heads % n_kv_heads == 0, W >= 0,
+ * max_ctx > 0) and lays out one ring per (layer, KV head, batch row), rings
+ * of equal capacity adjacent (one cache group per window level, Sec. 3.3).
+ * dev_arena: caller-owned device memory of arena_bytes >= hwkv_required_bytes
+ * (the cache does not free it), or NULL to let the library cudaMalloc it.
+ * The rings and workspace are zero-filled on `cuda_stream` before return
+ * completes (this call synchronizes that stream). Every layer starts with
+ * t = 0 tokens. On success *out owns the cache; release with hwkv_free.
+ */
+HWKV_API hwkv_status hwkv_alloc(const hwkv_policy* policy, void* dev_arena, size_t arena_bytes,
+                       void* cuda_stream, hwkv_cache** out);
+
+/* Releases the cache (and the arena if the library allocated it). NULL is a no-op. */
+HWKV_API hwkv_status hwkv_free(hwkv_cache* cache);
+
+/*
+ * Append/wrap (Sec. 3.3: a head keeps only its latest W states). Writes the
+ * n new tokens at positions t .. t+n-1 of `layer` into every KV head's ring,
+ * position p going to slot p mod cap; only the last min(n, cap) of them are
+ * written (earlier ones would be overwritten within the same call). Then t += n.
+ *   k, v: [batch, n, n_kv_heads, head_dim] bf16, device.
+ * n == 0 is a no-op. Fails with HWKV_ECAPACITY if t + n > max_ctx.
+ */
+HWKV_API hwkv_status hwkv_append(hwkv_cache* cache, int32_t layer, const void* k, const void* v,
+                        int64_t n, void* cuda_stream);
+
+/*
+ * Window-limited causal prefill of one chunk (Sec. 3.2, Eq. conditional-
+ * attention-weight and Eq. conditional-attention; the chunked prompt pass of
+ * App. "Experimental Protocol"). For the chunk at positions t0 .. t0+n-1
+ * (t0 = the layer's current t): query row p of query head q attends to the
+ * keys of KV head q/G at positions [max(0, p-W+1), p], taken from the ring
+ * (positions < t0) and from this chunk (positions >= t0), with logits
+ * scale * q.k. Then the chunk's K/V are appended as by hwkv_append.
+ *   q:   [batch, n, n_q_heads, head_dim] bf16
+ *   k,v: [batch, n, n_kv_heads, head_dim] bf16
+ *   out: [batch, n, n_q_heads, head_dim] fp32, the per-head outputs
+ *        concatenated in head order (pre-gate layout, Sec. 3.3).
+ * Because attention runs before the write, a ring of capacity exactly W
+ * serves chunks longer than W. Fails with HWKV_ECAPACITY as hwkv_append.
+ */
+HWKV_API hwkv_status hwkv_prefill(hwkv_cache* cache, int32_t layer, const void* q, const void* k,
+                         const void* v, int64_t n, float scale, float* out, void* cuda_stream);
+
+/*
+ * Decode attention (Sec. 3.2 at the newest position; Sec. 3.3 graph routing):
+ * the query at position p = t-1 (the token the caller appended last) of each
+ * query head attends over every resident slot of its KV head's ring, i.e.
+ * positions [max(0, t-W), t-1], with logits scale * q.k. Work is split over
+ * the rings in equal-length tiles (split count per head follows its resident
+ * length), each tile yields partial (max, sum, output) and a log-sum-exp merge
+ * combines them.
+ *   q:   [batch, n_q_heads, head_dim] bf16
+ *   out: [batch, n_q_heads, head_dim] fp32
+ * Fails with HWKV_EINVAL if the layer holds no tokens.
+ */
+HWKV_API hwkv_status hwkv_decode_attn(hwkv_cache* cache, int32_t layer, const void* q, float scale,
+                             float* out, void* cuda_stream);
+
+/*
+ * Resident K+V bytes (Sec. 3.1, Eq. nominal-storage with C = t, bf16 K and V,
+ * times batch): sum over KV heads of batch * min(cap, t) * head_dim * 2 * 2,
+ * for one layer, or summed over all layers when layer == -1. Host-only.
+ */
+HWKV_API hwkv_status hwkv_residency_bytes(const hwkv_cache* cache, int32_t layer, uint64_t* bytes);
+
+/* Bytes of ring storage allocated (sum of batch * cap * head_dim * 4); layer -1 = all. */
+HWKV_API hwkv_status hwkv_allocated_ring_bytes(const hwkv_cache* cache, int32_t layer, uint64_t* bytes);
+
+/* Tokens held by `layer` so far (its t). */
+HWKV_API hwkv_status hwkv_seq_len(const hwkv_cache* cache, int32_t layer, int64_t* t);
+
+/* Ring capacity of (layer, kv_head): min(W, max_ctx), or max_ctx for full. */
+HWKV_API hwkv_status hwkv_ring_capacity(const hwkv_cache* cache, int32_t layer, int32_t kv_head,
+                               int64_t* cap);
+
+/*
+ * Copies the ring of (layer, batch row b, kv_head) to host buffers
+ * k_host, v_host of cap * head_dim bf16 each (slot-major). Synchronizes the
+ * device. For tests and debugging.
+ */
+HWKV_API hwkv_status hwkv_debug_copy_ring(const hwkv_cache* cache, int32_t layer, int32_t b,
+                                 int32_t kv_head, void* k_host, void* v_host);
+
+/*
+ * Synchronizes the device and reads the cache's kernel error word; returns
+ * HWKV_EKERNEL (and clears the word) if a kernel gave up on a bounded wait or
+ * saw an inconsistent index, else HWKV_OK.
+ */
+HWKV_API hwkv_status hwkv_sync_check(hwkv_cache* cache);
+
+/* Message of the last failure on this thread ("" if none). */
+HWKV_API const char* hwkv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HWKV_H */

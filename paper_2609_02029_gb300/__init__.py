@@ -1,0 +1,191 @@
+"""Per-head-window KV cache attention for GB300 (HeadWiseKV grouped-cache hot path).
+
+Thin ctypes binding over ``libhwkv.so`` (C ABI in ``include/hwkv.h``). Every
+function here has the name of the C entry point it calls and only marshals
+arguments: device pointers may be passed as integers or as CUDA tensors
+(their ``data_ptr()``), streams as integers or ``torch.cuda.Stream``. All
+computation happens in the library's CUDA kernels; if the library is missing
+the import fails -- there is no fallback.
+"""
+import ctypes
+import os
+import re
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libhwkv.so")
+HEADER = os.path.join(os.path.dirname(_HERE), "include", "hwkv.h")
+
+HWKV_OK, HWKV_EINVAL, HWKV_ENOMEM, HWKV_ECAPACITY = 0, 1, 2, 3
+HWKV_ECUDA, HWKV_EKERNEL, HWKV_EUNSUPPORTED = 4, 5, 6
+HWKV_WINDOW_FULL = 0
+STATUS_NAMES = {0: "HWKV_OK", 1: "HWKV_EINVAL", 2: "HWKV_ENOMEM", 3: "HWKV_ECAPACITY",
+                4: "HWKV_ECUDA", 5: "HWKV_EKERNEL", 6: "HWKV_EUNSUPPORTED"}
+
+
+class HwkvError(RuntimeError):
+    def __init__(self, status, message):
+        super().__init__("%s: %s" % (STATUS_NAMES.get(status, status), message))
+        self.status = status
+
+
+class hwkv_policy(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("batch", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("max_ctx", ctypes.c_int64), ("windows", ctypes.POINTER(ctypes.c_int64))]
+
+
+def make_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, max_ctx, windows):
+    """hwkv_policy with its windows array ([n_layers * n_kv_heads] int64, 0 = full)
+    kept alive on the returned object."""
+    w = np.ascontiguousarray(np.asarray(windows, dtype=np.int64).ravel())
+    pol = hwkv_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, 0, max_ctx,
+                      w.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)))
+    pol._windows_keepalive = w
+    return pol
+
+
+_lib = None
+_vp, _i32, _i64, _u64p = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.POINTER(ctypes.c_uint64)
+
+
+def lib():
+    """The loaded libhwkv.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError("libhwkv.so not built: run `python -c 'import __graft_entry__ as g; "
+                              "g.build()'` (needs nvcc for sm_103a)")
+        L = ctypes.CDLL(LIB_PATH)
+        pp = ctypes.POINTER(hwkv_policy)
+        sig = {
+            "hwkv_required_bytes": [pp, ctypes.POINTER(ctypes.c_size_t)],
+            "hwkv_alloc": [pp, _vp, ctypes.c_size_t, _vp, ctypes.POINTER(_vp)],
+            "hwkv_free": [_vp],
+            "hwkv_append": [_vp, _i32, _vp, _vp, _i64, _vp],
+            "hwkv_prefill": [_vp, _i32, _vp, _vp, _vp, _i64, ctypes.c_float, _vp, _vp],
+            "hwkv_decode_attn": [_vp, _i32, _vp, ctypes.c_float, _vp, _vp],
+            "hwkv_residency_bytes": [_vp, _i32, _u64p],
+            "hwkv_allocated_ring_bytes": [_vp, _i32, _u64p],
+            "hwkv_seq_len": [_vp, _i32, ctypes.POINTER(_i64)],
+            "hwkv_ring_capacity": [_vp, _i32, _i32, ctypes.POINTER(_i64)],
+            "hwkv_debug_copy_ring": [_vp, _i32, _i32, _i32, _vp, _vp],
+            "hwkv_sync_check": [_vp],
+        }
+        for name, args in sig.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = ctypes.c_int
+        L.hwkv_last_error.argtypes = []
+        L.hwkv_last_error.restype = ctypes.c_char_p
+        _lib = L
+    return _lib
+
+
+def declared_symbols():
+    """Entry points declared in include/hwkv.h."""
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"HWKV_API\s+[\w\s\*]*?\b(hwkv_\w+)\s*\(", text)))
+
+
+def hwkv_last_error():
+    return lib().hwkv_last_error().decode()
+
+
+def _check(status):
+    if status != HWKV_OK:
+        raise HwkvError(status, hwkv_last_error())
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        if not x.is_cuda:
+            raise ValueError("expected a CUDA tensor")
+        if not x.is_contiguous():
+            raise ValueError("expected a contiguous tensor")
+        return x.data_ptr()
+    raise TypeError("expected a device pointer or CUDA tensor, got %r" % type(x))
+
+
+def _stream(s):
+    if s is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def hwkv_required_bytes(policy):
+    n = ctypes.c_size_t(0)
+    _check(lib().hwkv_required_bytes(ctypes.byref(policy), ctypes.byref(n)))
+    return n.value
+
+
+def hwkv_alloc(policy, dev_arena=None, arena_bytes=0, stream=None):
+    """Returns the opaque cache handle (ctypes.c_void_p)."""
+    out = _vp()
+    _check(lib().hwkv_alloc(ctypes.byref(policy), _ptr(dev_arena), arena_bytes, _stream(stream),
+                            ctypes.byref(out)))
+    return out
+
+
+def hwkv_free(cache):
+    _check(lib().hwkv_free(cache))
+
+
+def hwkv_append(cache, layer, k, v, n, stream=None):
+    _check(lib().hwkv_append(cache, layer, _ptr(k), _ptr(v), n, _stream(stream)))
+
+
+def hwkv_prefill(cache, layer, q, k, v, n, scale, out, stream=None):
+    _check(lib().hwkv_prefill(cache, layer, _ptr(q), _ptr(k), _ptr(v), n, scale, _ptr(out),
+                              _stream(stream)))
+
+
+def hwkv_decode_attn(cache, layer, q, scale, out, stream=None):
+    _check(lib().hwkv_decode_attn(cache, layer, _ptr(q), scale, _ptr(out), _stream(stream)))
+
+
+def hwkv_residency_bytes(cache, layer=-1):
+    v = ctypes.c_uint64(0)
+    _check(lib().hwkv_residency_bytes(cache, layer, ctypes.byref(v)))
+    return v.value
+
+
+def hwkv_allocated_ring_bytes(cache, layer=-1):
+    v = ctypes.c_uint64(0)
+    _check(lib().hwkv_allocated_ring_bytes(cache, layer, ctypes.byref(v)))
+    return v.value
+
+
+def hwkv_seq_len(cache, layer):
+    v = ctypes.c_int64(0)
+    _check(lib().hwkv_seq_len(cache, layer, ctypes.byref(v)))
+    return v.value
+
+
+def hwkv_ring_capacity(cache, layer, kv_head):
+    v = ctypes.c_int64(0)
+    _check(lib().hwkv_ring_capacity(cache, layer, kv_head, ctypes.byref(v)))
+    return v.value
+
+
+def hwkv_debug_copy_ring(cache, layer, b, kv_head, head_dim):
+    """(K, V) of one ring as uint16 bf16 bit arrays [cap, head_dim]."""
+    cap = hwkv_ring_capacity(cache, layer, kv_head)
+    k = np.zeros((cap, head_dim), dtype=np.uint16)
+    v = np.zeros((cap, head_dim), dtype=np.uint16)
+    _check(lib().hwkv_debug_copy_ring(cache, layer, b, kv_head,
+                                      k.ctypes.data_as(_vp), v.ctypes.data_as(_vp)))
+    return k, v
+
+
+def hwkv_sync_check(cache):
+    _check(lib().hwkv_sync_check(cache))

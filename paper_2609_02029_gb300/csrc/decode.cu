@@ -1,0 +1,370 @@
+// decode.cu -- split-KV decode attention over per-head rings, and its
+// log-sum-exp combine (HeadWiseKV Sec. 3.2, Eq. conditional-attention-weight
+// and Eq. conditional-attention, evaluated at the newest position; Sec. 3.3:
+// each GQA query-head group reads its KV head's own slice).
+//
+// Work decomposition. For one layer, every (batch row b, KV head h) ring holds
+// n_h = min(t, cap_h) resident slots; after the append of token t-1 these are
+// exactly the positions J_{t-1}(W_h), so the softmax runs over all of them and
+// slot order does not matter. Rings are cut into tiles of equal length
+// (tile_len tokens, a multiple of 64), so a full-history head gets many tiles
+// and a short-window head few: the split count follows the resident length and
+// all window levels share one launch. A persistent grid walks the tile list.
+//
+// Inside a CTA: warp 4 is the producer -- one lane issues 2-D TMA loads of
+// 64-token stages of K and V (128-byte swizzle, one box per 64 channels) into
+// a STAGES-deep shared-memory ring guarded by full/empty mbarriers. Warps 0-3
+// consume 16 tokens of each stage:
+//   S^T[16 tok x 8 heads]  = K[16 x D] . Q^T[D x 8]        (mma m16n8k16, K as A)
+//   online softmax per head column (max / sum over warp shuffles)
+//   O^T[D x 8 heads]      += V^T[D x 16] . P^T[16 x 8]     (mma m16n8k16, V^T via ldmatrix.trans)
+// where P^T reaches the B-operand layout through movmatrix.trans. Up to 8 query
+// heads of a GQA group share every K/V byte read. Each warp leaves a partial
+// (max, sum, unnormalised output); the four warps merge theirs in shared memory
+// into one partial per tile, and the combine kernel merges the tiles of a head.
+#include "hwkv_internal.cuh"
+
+namespace hwkv {
+
+namespace {
+
+struct TileInfo {
+  int b, h;
+  int64_t start;  // first slot of the tile
+  int len;        // slots in the tile (>= 1)
+  int64_t k_row, v_row;
+};
+
+__device__ __forceinline__ TileInfo locate_tile(const DecodeParams& p, int tile) {
+  TileInfo ti;
+  ti.b = tile / p.tiles_per_b;
+  const int lt = tile - ti.b * p.tiles_per_b;
+  int h = 0;
+  while (h + 1 < p.n_units && lt >= p.u[h].tile_begin + p.u[h].n_tiles) ++h;
+  ti.h = h;
+  const DecodeUnit& u = p.u[h];
+  const int i = lt - u.tile_begin;
+  ti.start = (int64_t)i * p.tile_len;
+  const int64_t rem = (int64_t)u.n_valid - ti.start;
+  ti.len = (int)(rem < p.tile_len ? rem : p.tile_len);
+  ti.k_row = u.k_row0 + (int64_t)ti.b * u.cap + ti.start;
+  ti.v_row = u.v_row0 + (int64_t)ti.b * u.cap + ti.start;
+  return ti;
+}
+
+// named barrier of the four consumer warps (the producer warp does not take part)
+__device__ __forceinline__ void consumer_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kDecodeWarps * 32) : "memory");
+}
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+template <int D>
+struct DecodeCfg {
+  static constexpr int kSlabs = D / 64;
+  static constexpr int kTileBytes = kSlabs * kSlabBytes;  // 64 tokens of K (or V)
+  static constexpr int kStageBytes = 2 * kTileBytes;
+  static constexpr int kStages = D == 256 ? 3 : (D == 128 ? 6 : 8);
+  static constexpr int kRedLd = D + 4;  // padded row of the cross-warp merge area (floats)
+  static constexpr int kRedBytes = kDecodeWarps * kMaxGroup * kRedLd * 4;
+  static constexpr int kMlBytes = kDecodeWarps * kMaxGroup * 8;
+  static constexpr int kSmem = kStages * kStageBytes + kRedBytes + kMlBytes + 2 * kStages * 8 + 1024;
+};
+
+}  // namespace
+
+template <int D>
+__global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
+    decode_split_kernel(const __grid_constant__ CUtensorMap kv_map, const DecodeParams p) {
+  using C = DecodeCfg<D>;
+  constexpr int STAGES = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  float* red_o = reinterpret_cast<float*>(smem + STAGES * C::kStageBytes);
+  float2* red_ml = reinterpret_cast<float2*>(smem + STAGES * C::kStageBytes + C::kRedBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::kStageBytes + C::kRedBytes +
+                                               C::kMlBytes);
+  uint64_t* empty = full + STAGES;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kDecodeWarps);
+    }
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  if (warp == kDecodeWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane != 0) return;
+    prefetch_tensormap(&kv_map);
+    uint32_t it = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; ok && tile < p.n_tiles; tile += gridDim.x) {
+      const TileInfo ti = locate_tile(p, tile);
+      const int n_st = (ti.len + kStageTokens - 1) / kStageTokens;
+      for (int st = 0; st < n_st; ++st, ++it) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1u;
+        if (!mbar_wait_bounded(&empty[s], ph ^ 1u, p.err)) {
+          ok = false;
+          break;
+        }
+        uint8_t* kdst = smem + s * C::kStageBytes;
+        uint8_t* vdst = kdst + C::kTileBytes;
+        mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+        const int32_t krow = (int32_t)(ti.k_row + (int64_t)st * kStageTokens);
+        const int32_t vrow = (int32_t)(ti.v_row + (int64_t)st * kStageTokens);
+#pragma unroll
+        for (int sl = 0; sl < C::kSlabs; ++sl)
+          tma_load_2d(kdst + sl * kSlabBytes, &kv_map, sl * 64, krow, &full[s]);
+#pragma unroll
+        for (int sl = 0; sl < C::kSlabs; ++sl)
+          tma_load_2d(vdst + sl * kSlabBytes, &kv_map, sl * 64, vrow, &full[s]);
+      }
+    }
+    if (!ok) {
+      // let the copies already issued land before the CTA's shared memory goes away
+      const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
+      for (uint32_t j = first; j < it; ++j)
+        mbar_wait_bounded(&full[j % STAGES], (j / STAGES) & 1u, p.err);
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  const int w = warp;
+  const int qn = lane >> 2;        // query head of this lane's Q^T fragment column
+  const int qk = (lane & 3) * 2;   // channel pair within a 16-channel step
+  const float c = p.scale_log2;
+  uint32_t it = 0;
+  // Once a bounded wait gives up, this warp stops waiting and computing but
+  // keeps walking the same tile/stage sequence, so every consumer warp still
+  // reaches the same named barriers.
+  bool aborted = false;
+
+  for (int tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x) {
+    const TileInfo ti = locate_tile(p, tile);
+    const int n_st = (ti.len + kStageTokens - 1) / kStageTokens;
+
+    // Q^T as mma B fragments: b0 = channels 16kk + qk + {0,1}, b1 = +8; column = head qn
+    uint32_t qf[D / 16][2];
+    {
+      const bool qv = qn < p.group;
+      const __nv_bfloat16* qrow =
+          p.q + ((int64_t)ti.b * p.n_q_heads + (int64_t)ti.h * p.group + (qv ? qn : 0)) * D;
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        qf[kk][0] = qv ? *reinterpret_cast<const uint32_t*>(qrow + kk * 16 + qk) : 0u;
+        qf[kk][1] = qv ? *reinterpret_cast<const uint32_t*>(qrow + kk * 16 + 8 + qk) : 0u;
+      }
+    }
+
+    float o[D / 16][4];
+#pragma unroll
+    for (int mt = 0; mt < D / 16; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+    float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
+
+    for (int st = 0; st < n_st; ++st, ++it) {
+      const int s = it % STAGES;
+      const uint32_t ph = (it / STAGES) & 1u;
+      if (!aborted && !mbar_wait_bounded(&full[s], ph, p.err)) aborted = true;
+      if (aborted) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[s]);
+        continue;
+      }
+      const uint32_t kbase = smem_u32(smem + s * C::kStageBytes);
+      const uint32_t vbase = kbase + C::kTileBytes;
+
+      // S^T = K . Q^T  (two accumulators to shorten the dependent mma chain)
+      float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+      {
+        const int r = w * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+        const int csel = lane >> 4;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4(kbase + (kk >> 2) * kSlabBytes + swz128(r, (kk & 3) * 2 + csel), a0, a1, a2,
+                  a3);
+          if (kk & 1)
+            mma_bf16_16816(sb, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+          else
+            mma_bf16_16816(sa, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+        }
+      }
+      float s0 = sa[0] + sb[0], s1 = sa[1] + sb[1], s2 = sa[2] + sb[2], s3 = sa[3] + sb[3];
+      const int tok = st * kStageTokens + w * 16 + (lane >> 2);
+      if (tok >= ti.len) s0 = s1 = -INFINITY;
+      if (tok + 8 >= ti.len) s2 = s3 = -INFINITY;
+
+      // online softmax; this lane owns head columns qk (A) and qk+1 (B)
+      float xA = fmaxf(s0, s2), xB = fmaxf(s1, s3);
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+        xA = fmaxf(xA, __shfl_xor_sync(0xffffffffu, xA, off));
+        xB = fmaxf(xB, __shfl_xor_sync(0xffffffffu, xB, off));
+      }
+      const float nA = fmaxf(mA, xA), nB = fmaxf(mB, xB);
+      const float uA = nA == -INFINITY ? 0.f : nA;
+      const float uB = nB == -INFINITY ? 0.f : nB;
+      const float alA = ex2((mA - uA) * c), alB = ex2((mB - uB) * c);
+      const float p0 = ex2((s0 - uA) * c), p1 = ex2((s1 - uB) * c);
+      const float p2 = ex2((s2 - uA) * c), p3 = ex2((s3 - uB) * c);
+      lA = lA * alA + p0 + p2;
+      lB = lB * alB + p1 + p3;
+      mA = nA;
+      mB = nB;
+      if (__any_sync(0xffffffffu, alA != 1.f || alB != 1.f)) {
+#pragma unroll
+        for (int mt = 0; mt < D / 16; ++mt) {
+          o[mt][0] *= alA;
+          o[mt][1] *= alB;
+          o[mt][2] *= alA;
+          o[mt][3] *= alB;
+        }
+      }
+      const uint32_t pb0 = movmatrix_trans(pack_bf16(p0, p1));
+      const uint32_t pb1 = movmatrix_trans(pack_bf16(p2, p3));
+
+      // O^T += V^T . P^T
+      {
+        const int mi = lane >> 3;
+        const int r = w * 16 + (lane & 7) + (mi >> 1) * 8;
+        const int csel = mi & 1;
+#pragma unroll
+        for (int mt = 0; mt < D / 16; ++mt) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4_t(vbase + (mt >> 2) * kSlabBytes + swz128(r, (mt & 3) * 2 + csel), a0, a1, a2,
+                    a3);
+          mma_bf16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[s]);
+    }
+
+    // ---- merge the four warps' partials of this tile in shared memory
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      lA += __shfl_xor_sync(0xffffffffu, lA, off);
+      lB += __shfl_xor_sync(0xffffffffu, lB, off);
+    }
+    consumer_sync();  // previous tile's merge has been read
+    {
+      float* ro = red_o + (size_t)w * kMaxGroup * C::kRedLd;
+#pragma unroll
+      for (int mt = 0; mt < D / 16; ++mt) {
+        const int dim = mt * 16 + (lane >> 2);
+        ro[qk * C::kRedLd + dim] = o[mt][0];
+        ro[(qk + 1) * C::kRedLd + dim] = o[mt][1];
+        ro[qk * C::kRedLd + dim + 8] = o[mt][2];
+        ro[(qk + 1) * C::kRedLd + dim + 8] = o[mt][3];
+      }
+      if (lane < 4) {
+        red_ml[w * kMaxGroup + qk] = make_float2(mA, lA);
+        red_ml[w * kMaxGroup + qk + 1] = make_float2(mB, lB);
+      }
+    }
+    consumer_sync();
+    {
+      float* po = p.part_o + (int64_t)tile * kMaxGroup * D;
+      for (int n = 0; n < p.group; ++n) {
+        float M = -INFINITY;
+#pragma unroll
+        for (int ww = 0; ww < kDecodeWarps; ++ww) M = fmaxf(M, red_ml[ww * kMaxGroup + n].x);
+        float e[kDecodeWarps], L = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < kDecodeWarps; ++ww) {
+          const float2 ml = red_ml[ww * kMaxGroup + n];
+          e[ww] = ml.x == -INFINITY ? 0.f : ex2((ml.x - M) * c);
+          L += e[ww] * ml.y;
+        }
+        for (int i = w * (D / kDecodeWarps) + lane; i < (w + 1) * (D / kDecodeWarps); i += 32) {
+          float acc = 0.f;
+#pragma unroll
+          for (int ww = 0; ww < kDecodeWarps; ++ww)
+            acc += e[ww] * red_o[((size_t)ww * kMaxGroup + n) * C::kRedLd + i];
+          po[(int64_t)n * D + i] = acc;
+        }
+        if (w == 0 && lane == 0) p.part_ml[(int64_t)tile * kMaxGroup + n] = make_float2(M, L);
+      }
+    }
+  }
+}
+
+// Log-sum-exp merge of the tile partials of one (batch row, KV head):
+// o = sum_i 2^{(m_i - M) c} o_i / sum_i 2^{(m_i - M) c} l_i, M = max_i m_i,
+// over the tiles in their fixed order (deterministic).
+template <int D>
+__global__ void __launch_bounds__(D) decode_combine_kernel(const DecodeParams p) {
+  const int b = blockIdx.x / p.n_units;
+  const int h = blockIdx.x - b * p.n_units;
+  const int i = threadIdx.x;
+  const DecodeUnit& u = p.u[h];
+  const int64_t tile0 = (int64_t)b * p.tiles_per_b + u.tile_begin;
+  const int n_t = u.n_tiles;
+  const float c = p.scale_log2;
+  for (int n = 0; n < p.group; ++n) {
+    float M = -INFINITY;
+    for (int j = 0; j < n_t; ++j) M = fmaxf(M, p.part_ml[(tile0 + j) * kMaxGroup + n].x);
+    float num = 0.f, den = 0.f;
+    for (int j = 0; j < n_t; ++j) {
+      const float2 ml = p.part_ml[(tile0 + j) * kMaxGroup + n];
+      if (ml.x == -INFINITY) continue;
+      const float wgt = ex2((ml.x - M) * c);
+      num += wgt * p.part_o[((tile0 + j) * kMaxGroup + n) * D + i];
+      den += wgt * ml.y;
+    }
+    p.out[((int64_t)b * p.n_q_heads + (int64_t)h * p.group + n) * D + i] = num / den;
+  }
+}
+
+int decode_smem_bytes(int head_dim) {
+  switch (head_dim) {
+    case 64: return DecodeCfg<64>::kSmem;
+    case 128: return DecodeCfg<128>::kSmem;
+    case 256: return DecodeCfg<256>::kSmem;
+    default: return -1;
+  }
+}
+
+template <int D>
+static cudaError_t launch_decode_t(const DecodeParams& p, const CUtensorMap& map, int grid,
+                                   cudaStream_t s) {
+  const int smem = DecodeCfg<D>::kSmem;
+  cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  decode_split_kernel<D><<<grid, (kDecodeWarps + 1) * 32, smem, s>>>(map, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& map, int head_dim, int grid,
+                          cudaStream_t s) {
+  switch (head_dim) {
+    case 64: return launch_decode_t<64>(p, map, grid, s);
+    case 128: return launch_decode_t<128>(p, map, grid, s);
+    case 256: return launch_decode_t<256>(p, map, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s) {
+  const int grid = p.batch * p.n_units;
+  switch (head_dim) {
+    case 64: decode_combine_kernel<64><<<grid, 64, 0, s>>>(p); break;
+    case 128: decode_combine_kernel<128><<<grid, 128, 0, s>>>(p); break;
+    case 256: decode_combine_kernel<256><<<grid, 256, 0, s>>>(p); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace hwkv

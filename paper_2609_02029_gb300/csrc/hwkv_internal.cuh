@@ -1,0 +1,234 @@
+// hwkv_internal.cuh -- shared device helpers and launch parameter blocks of libhwkv.
+//
+// Inline PTX for sm_103a: mbarrier (with bounded waits that report through an
+// error word instead of spinning forever), TMA tensor loads, ldmatrix, warp-level
+// bf16 mma and movmatrix.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace hwkv {
+
+constexpr int kMaxKvHeads = 64;
+constexpr int kMaxGroup = 8;          // query heads per KV head handled by one mma n-tile
+constexpr int kDecodeWarps = 4;       // consumer warps per decode CTA
+constexpr int kStageTokens = 64;      // tokens per pipeline stage (16 per consumer warp)
+constexpr int kSlabBytes = 64 * 128;  // one TMA box: 64 rows x 128 B (64 bf16)
+
+// error word bits (set with atomicOr, read by hwkv_sync_check)
+constexpr int kErrWaitTimeout = 1;
+constexpr int kErrBadIndex = 2;
+
+// ------------------------------------------------------------------ decode
+struct DecodeUnit {
+  int64_t k_row0;   // arena row of (this KV head, batch row 0) in the K region
+  int64_t v_row0;   // same in the V region
+  int64_t cap;      // ring capacity; batch row b starts at row0 + b * cap
+  int32_t n_valid;  // resident slots: min(t, cap)
+  int32_t n_tiles;  // tiles this head's ring is split into, per batch row
+  int32_t tile_begin;  // first tile of this head within one batch row's tile list
+  int32_t pad;
+};
+
+struct DecodeParams {
+  int32_t n_units;      // KV heads of the layer
+  int32_t batch;
+  int32_t group;        // G = n_q_heads / n_kv_heads
+  int32_t n_q_heads;
+  int32_t tile_len;     // tokens per tile, multiple of kStageTokens
+  int32_t tiles_per_b;  // sum of n_tiles over heads
+  int32_t n_tiles;      // batch * tiles_per_b
+  float scale_log2;     // scale * log2(e)
+  const __nv_bfloat16* q;  // [batch][n_q_heads][D]
+  float* part_o;           // [n_tiles * kDecodeWarps][D][kMaxGroup]
+  float2* part_ml;         // [n_tiles * kDecodeWarps][kMaxGroup]  (max, sum)
+  float* out;              // [batch][n_q_heads][D]
+  int* err;
+  DecodeUnit u[kMaxKvHeads];
+};
+
+// ------------------------------------------------------------------ append
+struct AppendUnit {
+  int64_t k_row0, v_row0, cap;
+};
+
+struct AppendParams {
+  int32_t n_units, batch;
+  int64_t t0;      // position of the first new token
+  int64_t n;       // new tokens
+  int64_t d;       // head_dim
+  const __nv_bfloat16* k;  // [batch][n][n_units][d]
+  const __nv_bfloat16* v;
+  __nv_bfloat16* k_arena;  // row r at k_arena + r * d
+  __nv_bfloat16* v_arena;
+  AppendUnit u[kMaxKvHeads];
+};
+
+// ------------------------------------------------------------------ prefill
+struct PrefillUnit {
+  int64_t k_row0, v_row0, cap;
+  int64_t window;  // 0 = full
+};
+
+struct PrefillParams {
+  int32_t n_units, batch, group, n_q_heads;
+  int64_t t0;  // first chunk position (tokens already in the cache)
+  int64_t n;   // chunk length
+  float scale_log2;
+  const __nv_bfloat16* q;   // [batch][n][n_q_heads][D]
+  const __nv_bfloat16* k;   // [batch][n][n_units][D]
+  const __nv_bfloat16* v;
+  const __nv_bfloat16* k_arena;
+  const __nv_bfloat16* v_arena;
+  float* out;               // [batch][n][n_q_heads][D]
+  int* err;
+  PrefillUnit u[kMaxKvHeads];
+};
+
+// launchers (defined in the kernel translation units); return cudaGetLastError()
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& kv_map, int head_dim,
+                          int grid, cudaStream_t s);
+cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s);
+cudaError_t launch_prefill(const PrefillParams& p, int head_dim, cudaStream_t s);
+int decode_smem_bytes(int head_dim);
+
+// ------------------------------------------------------------ device PTX
+#if defined(__CUDACC__)
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Waits for the phase of `parity` to complete, giving up after ~2 s.
+// Returns false (and sets the error word) on timeout.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, int* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 0u && globaltimer_ns() - t0 > 2000000000ull) {
+      atomicOr(err, kErrWaitTimeout);
+      return false;
+    }
+  }
+}
+
+// 2-D TMA tile load (x = column in elements, y = row) completing on `bar`
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int32_t x,
+                                            int32_t y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];"
+               : "=r"(r0), "=r"(r1)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];"
+               : "=r"(r0), "=r"(r1)
+               : "r"(addr));
+}
+
+// D = A(16x16, row) * B(16x8, col) + D, bf16 inputs, fp32 accumulate
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
+                                               uint32_t a2, uint32_t a3, uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// (lo, hi) -> bf16x2 with lo in the low half, round to nearest even
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// byte offset of 16-byte chunk `c` (0..7) of row `r` inside a 128B-swizzled slab
+__device__ __forceinline__ uint32_t swz128(int r, int c) {
+  return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4));
+}
+
+#endif  // __CUDACC__
+
+}  // namespace hwkv

@@ -1,0 +1,485 @@
+// runtime.cu -- host side of libhwkv: the C ABI of include/hwkv.h.
+//
+// Policy -> physical layout (HeadWiseKV Sec. 3.3 and App. "Runtime
+// Realization": storage partitioned into (window, KV head) groups; each
+// configured head owns a slice sized to its window, disjoint per layer).
+// Here every (layer, KV head, batch row) owns one K ring and one V ring of
+// cap = min(W, max_ctx) rows of head_dim bf16; rings of the same capacity
+// (one window level) are adjacent in one arena, K region first, then the V
+// region in the same order, then the decode workspace.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include <cudaTypedefs.h>
+
+#include "../../include/hwkv.h"
+#include "hwkv_internal.cuh"
+
+using namespace hwkv;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+hwkv_status fail(hwkv_status st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+hwkv_status fail(hwkv_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+hwkv_status ok() {
+  g_last_error.clear();
+  return HWKV_OK;
+}
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct Unit {
+  int64_t window;  // effective: 0 = full
+  int64_t cap;
+  int64_t k_row0, v_row0;
+};
+
+struct Layout {
+  std::vector<Unit> units;  // [layer * n_kv_heads + h]
+  int64_t rows = 0;         // K rows (= V rows)
+  size_t ring_bytes = 0;    // K + V
+  size_t part_o_off = 0, part_ml_off = 0, err_off = 0, total = 0;
+  int max_tiles = 0;
+};
+
+hwkv_status validate(const hwkv_policy* p) {
+  if (!p) return fail(HWKV_EINVAL, "policy is NULL");
+  if (p->n_layers <= 0 || p->n_kv_heads <= 0 || p->n_q_heads <= 0 || p->batch <= 0 ||
+      p->head_dim <= 0 || p->max_ctx <= 0)
+    return fail(HWKV_EINVAL, "policy sizes must be positive");
+  if (p->n_q_heads % p->n_kv_heads != 0)
+    return fail(HWKV_EINVAL, "n_q_heads (%d) must be a multiple of n_kv_heads (%d)",
+                p->n_q_heads, p->n_kv_heads);
+  if (!p->windows) return fail(HWKV_EINVAL, "policy windows is NULL");
+  for (int64_t i = 0; i < (int64_t)p->n_layers * p->n_kv_heads; ++i)
+    if (p->windows[i] < 0)
+      return fail(HWKV_EINVAL, "window of (layer %lld, kv head %lld) is negative",
+                  (long long)(i / p->n_kv_heads), (long long)(i % p->n_kv_heads));
+  if (p->head_dim != 64 && p->head_dim != 128 && p->head_dim != 256)
+    return fail(HWKV_EUNSUPPORTED, "head_dim %d not built (64, 128, 256)", p->head_dim);
+  if (p->n_q_heads / p->n_kv_heads > kMaxGroup)
+    return fail(HWKV_EUNSUPPORTED, "GQA group %d > %d", p->n_q_heads / p->n_kv_heads, kMaxGroup);
+  if (p->n_kv_heads > kMaxKvHeads)
+    return fail(HWKV_EUNSUPPORTED, "n_kv_heads %d > %d", p->n_kv_heads, kMaxKvHeads);
+  if (p->batch > 256) return fail(HWKV_EUNSUPPORTED, "batch %d > 256", p->batch);
+  return HWKV_OK;
+}
+
+Layout make_layout(const hwkv_policy* p) {
+  Layout L;
+  const int nu = p->n_layers * p->n_kv_heads;
+  L.units.resize(nu);
+  for (int i = 0; i < nu; ++i) {
+    const int64_t W = p->windows[i];
+    Unit& u = L.units[i];
+    u.window = (W == HWKV_WINDOW_FULL || W >= p->max_ctx) ? 0 : W;  // w >= C is full (Sec. 3.1)
+    u.cap = u.window == 0 ? p->max_ctx : u.window;
+  }
+  // group by level: larger capacity first, then layer, then head
+  std::vector<int> order(nu);
+  for (int i = 0; i < nu; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int a, int b) { return L.units[a].cap > L.units[b].cap; });
+  int64_t row = 0;
+  for (int i : order) {
+    L.units[i].k_row0 = row;
+    row += L.units[i].cap * p->batch;
+  }
+  L.rows = row;
+  for (auto& u : L.units) u.v_row0 = u.k_row0 + L.rows;
+  const size_t row_bytes = (size_t)p->head_dim * 2;
+  L.ring_bytes = (size_t)(2 * L.rows) * row_bytes;
+  L.max_tiles = std::max(2048, 2 * p->batch * p->n_kv_heads);
+  L.part_o_off = align_up(L.ring_bytes, kAlign);
+  L.part_ml_off =
+      align_up(L.part_o_off + (size_t)L.max_tiles * kMaxGroup * p->head_dim * 4, kAlign);
+  L.err_off = align_up(L.part_ml_off + (size_t)L.max_tiles * kMaxGroup * 8, kAlign);
+  L.total = align_up(L.err_off + 64, kAlign);
+  return L;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  return fn;
+}
+
+}  // namespace
+
+struct hwkv_cache {
+  hwkv_policy pol;
+  std::vector<int64_t> windows;
+  Layout lay;
+  std::vector<int64_t> t;  // tokens held, per layer
+  uint8_t* arena = nullptr;
+  bool owns_arena = false;
+  int num_sms = 0;
+  CUtensorMap kv_map;  // 2-D view of the K and V regions: [2 * rows][head_dim] bf16
+  __nv_bfloat16* k_base() const { return reinterpret_cast<__nv_bfloat16*>(arena); }
+  __nv_bfloat16* v_base() const { return k_base() + lay.rows * pol.head_dim; }
+  float* part_o() const { return reinterpret_cast<float*>(arena + lay.part_o_off); }
+  float2* part_ml() const { return reinterpret_cast<float2*>(arena + lay.part_ml_off); }
+  int* err() const { return reinterpret_cast<int*>(arena + lay.err_off); }
+};
+
+extern "C" {
+
+const char* hwkv_last_error(void) { return g_last_error.c_str(); }
+
+hwkv_status hwkv_required_bytes(const hwkv_policy* policy, size_t* arena_bytes) {
+  if (!arena_bytes) return fail(HWKV_EINVAL, "arena_bytes is NULL");
+  hwkv_status st = validate(policy);
+  if (st != HWKV_OK) return st;
+  *arena_bytes = make_layout(policy).total;
+  return ok();
+}
+
+hwkv_status hwkv_alloc(const hwkv_policy* policy, void* dev_arena, size_t arena_bytes,
+                       void* cuda_stream, hwkv_cache** out) {
+  if (!out) return fail(HWKV_EINVAL, "out is NULL");
+  *out = nullptr;
+  hwkv_status st = validate(policy);
+  if (st != HWKV_OK) return st;
+  Layout lay = make_layout(policy);
+  if (2 * lay.rows + kStageTokens >= (int64_t)INT32_MAX)
+    return fail(HWKV_EUNSUPPORTED, "ring rows %lld exceed the 2^31 TMA coordinate range",
+                (long long)(2 * lay.rows));
+  if (dev_arena && arena_bytes < lay.total)
+    return fail(HWKV_ENOMEM, "arena of %zu bytes < required %zu", arena_bytes, lay.total);
+  if (dev_arena && (reinterpret_cast<uintptr_t>(dev_arena) % kAlign) != 0)
+    return fail(HWKV_EINVAL, "dev_arena must be %zu-byte aligned", kAlign);
+  auto encode = get_encode();
+  if (!encode) return fail(HWKV_ECUDA, "cuTensorMapEncodeTiled entry point unavailable");
+
+  hwkv_cache* c = new hwkv_cache();
+  c->pol = *policy;
+  c->windows.assign(policy->windows, policy->windows + (size_t)policy->n_layers * policy->n_kv_heads);
+  c->pol.windows = c->windows.data();
+  c->lay = std::move(lay);
+  c->t.assign(policy->n_layers, 0);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) {
+    delete c;
+    return fail(HWKV_ECUDA, "device query failed: %s", cudaGetErrorString(e));
+  }
+  if (dev_arena) {
+    c->arena = static_cast<uint8_t*>(dev_arena);
+  } else {
+    e = cudaMalloc(reinterpret_cast<void**>(&c->arena), c->lay.total);
+    if (e != cudaSuccess) {
+      delete c;
+      return fail(HWKV_ENOMEM, "cudaMalloc(%zu) failed: %s", c->lay.total, cudaGetErrorString(e));
+    }
+    c->owns_arena = true;
+  }
+  e = cudaMemsetAsync(c->arena, 0, c->lay.total, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) {
+    if (c->owns_arena) cudaFree(c->arena);
+    delete c;
+    return fail(HWKV_ECUDA, "zero-fill failed: %s", cudaGetErrorString(e));
+  }
+  // one tensor map over both regions: rows of head_dim bf16, boxes of 64 rows x 64 channels
+  const cuuint64_t gdim[2] = {(cuuint64_t)c->pol.head_dim, (cuuint64_t)(2 * c->lay.rows)};
+  const cuuint64_t gstride[1] = {(cuuint64_t)c->pol.head_dim * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kStageTokens};
+  const cuuint32_t estride[2] = {1, 1};
+  CUresult r = encode(&c->kv_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->arena, gdim, gstride,
+                      box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (c->owns_arena) cudaFree(c->arena);
+    delete c;
+    return fail(HWKV_ECUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  }
+  *out = c;
+  return ok();
+}
+
+hwkv_status hwkv_free(hwkv_cache* c) {
+  if (!c) return ok();
+  if (c->owns_arena) cudaFree(c->arena);
+  delete c;
+  return ok();
+}
+
+static hwkv_status check_layer(const hwkv_cache* c, int32_t layer) {
+  if (!c) return fail(HWKV_EINVAL, "cache is NULL");
+  if (layer < 0 || layer >= c->pol.n_layers)
+    return fail(HWKV_EINVAL, "layer %d out of range [0, %d)", layer, c->pol.n_layers);
+  return HWKV_OK;
+}
+
+static AppendParams append_params(const hwkv_cache* c, int32_t layer, const void* k,
+                                  const void* v, int64_t n) {
+  AppendParams p{};
+  p.n_units = c->pol.n_kv_heads;
+  p.batch = c->pol.batch;
+  p.t0 = c->t[layer];
+  p.n = n;
+  p.d = c->pol.head_dim;
+  p.k = static_cast<const __nv_bfloat16*>(k);
+  p.v = static_cast<const __nv_bfloat16*>(v);
+  p.k_arena = c->k_base();
+  p.v_arena = c->k_base();  // V rows are addressed by v_row0, which already includes the K region
+  for (int h = 0; h < p.n_units; ++h) {
+    const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
+    p.u[h] = AppendUnit{u.k_row0, u.v_row0, u.cap};
+  }
+  return p;
+}
+
+hwkv_status hwkv_append(hwkv_cache* c, int32_t layer, const void* k, const void* v, int64_t n,
+                        void* cuda_stream) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (n < 0) return fail(HWKV_EINVAL, "n must be >= 0");
+  if (n == 0) return ok();
+  if (!k || !v) return fail(HWKV_EINVAL, "k/v is NULL");
+  if (c->t[layer] + n > c->pol.max_ctx)
+    return fail(HWKV_ECAPACITY, "layer %d: t=%lld + n=%lld exceeds max_ctx=%lld", layer,
+                (long long)c->t[layer], (long long)n, (long long)c->pol.max_ctx);
+  const AppendParams p = append_params(c, layer, k, v, n);
+  cudaError_t e = launch_append(p, static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "append launch: %s", cudaGetErrorString(e));
+  c->t[layer] += n;
+  return ok();
+}
+
+hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void* k,
+                         const void* v, int64_t n, float scale, float* out, void* cuda_stream) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (n < 0) return fail(HWKV_EINVAL, "n must be >= 0");
+  if (n == 0) return ok();
+  if (!q || !k || !v || !out) return fail(HWKV_EINVAL, "q/k/v/out is NULL");
+  if (c->t[layer] + n > c->pol.max_ctx)
+    return fail(HWKV_ECAPACITY, "layer %d: t=%lld + n=%lld exceeds max_ctx=%lld", layer,
+                (long long)c->t[layer], (long long)n, (long long)c->pol.max_ctx);
+  if (n > (int64_t)65535 * 64) return fail(HWKV_EUNSUPPORTED, "chunk of %lld tokens too long", (long long)n);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  PrefillParams p{};
+  p.n_units = c->pol.n_kv_heads;
+  p.batch = c->pol.batch;
+  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
+  p.n_q_heads = c->pol.n_q_heads;
+  p.t0 = c->t[layer];
+  p.n = n;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.k = static_cast<const __nv_bfloat16*>(k);
+  p.v = static_cast<const __nv_bfloat16*>(v);
+  p.k_arena = c->k_base();
+  p.v_arena = c->k_base();
+  p.out = out;
+  p.err = c->err();
+  for (int h = 0; h < p.n_units; ++h) {
+    const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
+    p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window};
+  }
+  cudaError_t e = launch_prefill(p, c->pol.head_dim, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "prefill launch: %s", cudaGetErrorString(e));
+  // attend first, then write the chunk's retained tokens (stream order)
+  const AppendParams ap = append_params(c, layer, k, v, n);
+  e = launch_append(ap, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "append launch: %s", cudaGetErrorString(e));
+  c->t[layer] += n;
+  return ok();
+}
+
+// Decode tile plan: equal-length tiles (multiple of 64 tokens) over every
+// (batch row, KV head) ring. The length is chosen to balance the persistent
+// grid: minimise (tiles per CTA) x (tile length + a fixed per-tile cost).
+static void plan_decode(const hwkv_cache* c, int32_t layer, DecodeParams& p, int& grid) {
+  const int H = c->pol.n_kv_heads, B = c->pol.batch;
+  const int64_t t = c->t[layer];
+  int64_t n_valid[kMaxKvHeads];
+  int64_t longest = 0;
+  for (int h = 0; h < H; ++h) {
+    const Unit& u = c->lay.units[(size_t)layer * H + h];
+    n_valid[h] = std::min(t, u.cap);
+    longest = std::max(longest, n_valid[h]);
+  }
+  const int sms = std::max(1, c->num_sms);
+  auto count = [&](int64_t len) {
+    int64_t n = 0;
+    for (int h = 0; h < H; ++h) n += (n_valid[h] + len - 1) / len;
+    return n * B;
+  };
+  const int64_t per_tile_cost = 96;  // tokens-equivalent of a tile's fixed cost
+  int64_t best_len = 0;
+  double best = 0;
+  const int64_t max_len = std::max<int64_t>(64, (longest + 63) / 64 * 64);
+  for (int64_t len = 128; ; len = len < 1024 ? len + 64 : len + len / 8 / 64 * 64) {
+    const int64_t L = std::min(len, max_len);
+    const int64_t nt = count(L);
+    if (nt <= c->lay.max_tiles) {
+      const int64_t g = std::min<int64_t>(nt, sms);
+      const double cost = (double)((nt + g - 1) / g) * (double)(L + per_tile_cost);
+      if (best_len == 0 || cost < best) {
+        best = cost;
+        best_len = L;
+      }
+    }
+    if (L >= max_len) break;
+  }
+  if (best_len == 0) best_len = max_len;
+  p.tile_len = (int32_t)best_len;
+  int32_t begin = 0;
+  for (int h = 0; h < H; ++h) {
+    const Unit& u = c->lay.units[(size_t)layer * H + h];
+    DecodeUnit& du = p.u[h];
+    du.k_row0 = u.k_row0;
+    du.v_row0 = u.v_row0;
+    du.cap = u.cap;
+    du.n_valid = (int32_t)n_valid[h];
+    du.n_tiles = (int32_t)((n_valid[h] + best_len - 1) / best_len);
+    du.tile_begin = begin;
+    du.pad = 0;
+    begin += du.n_tiles;
+  }
+  p.tiles_per_b = begin;
+  p.n_tiles = begin * B;
+  grid = std::min(p.n_tiles, sms);
+}
+
+hwkv_status hwkv_decode_attn(hwkv_cache* c, int32_t layer, const void* q, float scale, float* out,
+                             void* cuda_stream) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (!q || !out) return fail(HWKV_EINVAL, "q/out is NULL");
+  if (c->t[layer] <= 0) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
+  if (c->t[layer] > INT32_MAX) return fail(HWKV_EUNSUPPORTED, "ring longer than 2^31");
+  DecodeParams p{};
+  p.n_units = c->pol.n_kv_heads;
+  p.batch = c->pol.batch;
+  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
+  p.n_q_heads = c->pol.n_q_heads;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.part_o = c->part_o();
+  p.part_ml = c->part_ml();
+  p.out = out;
+  p.err = c->err();
+  int grid = 0;
+  plan_decode(c, layer, p, grid);
+  if (p.n_tiles > c->lay.max_tiles)
+    return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = launch_decode(p, c->kv_map, c->pol.head_dim, grid, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
+  e = launch_decode_combine(p, c->pol.head_dim, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
+  return ok();
+}
+
+hwkv_status hwkv_residency_bytes(const hwkv_cache* c, int32_t layer, uint64_t* bytes) {
+  if (!c || !bytes) return fail(HWKV_EINVAL, "NULL argument");
+  if (layer < -1 || layer >= c->pol.n_layers) return fail(HWKV_EINVAL, "layer out of range");
+  const int H = c->pol.n_kv_heads;
+  const uint64_t per_token = (uint64_t)c->pol.head_dim * 2 * 2;  // d^K b^K + d^V b^V, bf16
+  uint64_t total = 0;
+  for (int l = 0; l < c->pol.n_layers; ++l) {
+    if (layer >= 0 && l != layer) continue;
+    for (int h = 0; h < H; ++h) {
+      const Unit& u = c->lay.units[(size_t)l * H + h];
+      total += (uint64_t)std::min(c->t[l], u.cap) * per_token * (uint64_t)c->pol.batch;
+    }
+  }
+  *bytes = total;
+  return ok();
+}
+
+hwkv_status hwkv_allocated_ring_bytes(const hwkv_cache* c, int32_t layer, uint64_t* bytes) {
+  if (!c || !bytes) return fail(HWKV_EINVAL, "NULL argument");
+  if (layer < -1 || layer >= c->pol.n_layers) return fail(HWKV_EINVAL, "layer out of range");
+  const int H = c->pol.n_kv_heads;
+  uint64_t total = 0;
+  for (int l = 0; l < c->pol.n_layers; ++l) {
+    if (layer >= 0 && l != layer) continue;
+    for (int h = 0; h < H; ++h)
+      total += (uint64_t)c->lay.units[(size_t)l * H + h].cap * c->pol.head_dim * 4 *
+               (uint64_t)c->pol.batch;
+  }
+  *bytes = total;
+  return ok();
+}
+
+hwkv_status hwkv_seq_len(const hwkv_cache* c, int32_t layer, int64_t* t) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (!t) return fail(HWKV_EINVAL, "t is NULL");
+  *t = c->t[layer];
+  return ok();
+}
+
+hwkv_status hwkv_ring_capacity(const hwkv_cache* c, int32_t layer, int32_t kv_head, int64_t* cap) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (kv_head < 0 || kv_head >= c->pol.n_kv_heads || !cap)
+    return fail(HWKV_EINVAL, "bad kv_head or NULL cap");
+  *cap = c->lay.units[(size_t)layer * c->pol.n_kv_heads + kv_head].cap;
+  return ok();
+}
+
+hwkv_status hwkv_debug_copy_ring(const hwkv_cache* c, int32_t layer, int32_t b, int32_t kv_head,
+                                 void* k_host, void* v_host) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (b < 0 || b >= c->pol.batch || kv_head < 0 || kv_head >= c->pol.n_kv_heads || !k_host ||
+      !v_host)
+    return fail(HWKV_EINVAL, "bad ring coordinates or NULL buffer");
+  const Unit& u = c->lay.units[(size_t)layer * c->pol.n_kv_heads + kv_head];
+  const size_t row = (size_t)c->pol.head_dim * 2;
+  const uint8_t* kb = c->arena + (size_t)(u.k_row0 + (int64_t)b * u.cap) * row;
+  const uint8_t* vb = c->arena + (size_t)(u.v_row0 + (int64_t)b * u.cap) * row;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpy(k_host, kb, (size_t)u.cap * row, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemcpy(v_host, vb, (size_t)u.cap * row, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "ring copy: %s", cudaGetErrorString(e));
+  return ok();
+}
+
+hwkv_status hwkv_sync_check(hwkv_cache* c) {
+  if (!c) return fail(HWKV_EINVAL, "cache is NULL");
+  int word = 0;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpy(&word, c->err(), sizeof word, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "sync: %s", cudaGetErrorString(e));
+  if (word != 0) {
+    cudaMemset(c->err(), 0, sizeof(int));
+    return fail(HWKV_EKERNEL, "kernel error word 0x%x (1 = bounded wait gave up, 2 = bad index)",
+                word);
+  }
+  return ok();
+}
+
+}  // extern "C"
