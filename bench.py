@@ -1,0 +1,605 @@
+"""Benchmark of the per-head-window KV decode path on GB300.
+
+One step = one decode step of every layer of the workload: for each layer,
+append the new token's K/V into every KV head's ring (hwkv_append), then
+split-KV decode attention of all query heads over the resident rings with the
+log-sum-exp combine (hwkv_decode_attn), plus the residency query
+(hwkv_residency_bytes). Inputs are seeded synthetic bf16 tensors from
+hwkv_gen with the workload's shapes; the prompt is filled (untimed) before.
+
+Prints one JSON line. `value` is decode tokens/s of the whole job (batch rows
+x steps / max-over-ranks time), inputs resident in HBM; `e2e` is the same
+metric with each step's q/k/v copied from pinned host memory and the outputs
+read back inside the timed region. `roofline` rates the decode kernel against
+the measured HBM copy bandwidth; `prefill` reports the window-limited prefill
+(64K prompt in 8K chunks) in TFLOP/s; `cpu_baseline` is the fp64 oracle on a
+bounded sample, on the host cores.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+    python bench.py --impl reference ...   # the oracle arm, on host cores
+"""
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from hwkv_gen import workloads  # noqa: E402
+
+NOMINAL_HBM_GBS = 8000.0
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(
+            d.get("bf16_tflops_sustained", d["bf16_tflops"])), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ------------------------------------------------------------------ ranks
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = os.environ.get("HWKV_BENCH_BACKEND", "nccl")
+        if backend == "nccl":
+            import torch
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    """Max of a float over all ranks (the job's time is its slowest rank)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            import tempfile
+            fd, self.path = tempfile.mkstemp(prefix="hwkv_clocks_", suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        rows = []
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) >= 9:
+                try:
+                    rows.append((float(f[1]), float(f[2]), f[5:9]))
+                except ValueError:
+                    pass
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r)
+                          if v.lower().startswith("active")})
+        sm = sorted(r[0] for r in rows)
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ------------------------------------------------------------ GPU decode
+def decode_bytes(wl, max_ctx, t):
+    """Algorithmic bytes of one decode launch per layer at length t: every
+    resident K/V row read once, batch x sum_h min(t, cap_h) x 4 d (q and out
+    are under 0.1 % and excluded)."""
+    per_layer = []
+    for layer in range(wl.n_layers):
+        s = 0
+        for h in range(wl.n_kv_heads):
+            W = wl.windows[layer * wl.n_kv_heads + h]
+            cap = max_ctx if (W == 0 or W >= max_ctx) else W
+            s += wl.batch * min(t, cap) * 4 * wl.head_dim
+        per_layer.append(s)
+    return per_layer
+
+
+def run_gpu(args, wl, world, rank, local):
+    import torch
+
+    import hwkv_gen
+    import paper_2609_02029_gb300 as hwkv
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    hwkv.lib()
+    stream = torch.cuda.current_stream(dev)  # every allocation and launch on one stream
+    s = stream.cuda_stream
+    g = hwkv_gen.desc(wl.seed + 1000003 * rank, wl.per_head_scale)  # each rank its own batch
+    L, B, Hq, Hkv, d = wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+    e2e_steps = min(args.steps, args.e2e_steps)
+    total_steps = args.warmup + args.steps + 2 + e2e_steps
+    prompt = wl.prompt
+    max_ctx = prompt + max(wl.decode_steps, total_steps)
+    scale = 1.0 / np.sqrt(d)
+
+    pol = hwkv.make_policy(L, Hkv, Hq, d, B, max_ctx, wl.windows)
+    nbytes = hwkv.hwkv_required_bytes(pol)
+    arena = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    cache = hwkv.hwkv_alloc(pol, arena, nbytes, s)
+
+    # prompt fill (untimed): generated chunks appended through the C ABI
+    chunk = 4096
+    kbuf = torch.empty((B, chunk, Hkv, d), dtype=torch.bfloat16, device=dev)
+    vbuf = torch.empty_like(kbuf)
+    for layer in range(L):
+        done = 0
+        while done < prompt:
+            n = min(chunk, prompt - done)
+            hwkv_gen.fill_device(g, hwkv_gen.K, layer, B, done, n, Hkv, d, kbuf.data_ptr(), s)
+            hwkv_gen.fill_device(g, hwkv_gen.V, layer, B, done, n, Hkv, d, vbuf.data_ptr(), s)
+            hwkv.hwkv_append(cache, layer, kbuf, vbuf, n, s)
+            done += n
+    del kbuf, vbuf
+
+    # per-step inputs (q of the new token, its K/V), pre-generated on the device
+    def gen_step(pos):
+        q = torch.empty((L, B, Hq, d), dtype=torch.bfloat16, device=dev)
+        k = torch.empty((L, B, 1, Hkv, d), dtype=torch.bfloat16, device=dev)
+        v = torch.empty_like(k)
+        for layer in range(L):
+            hwkv_gen.fill_device(g, hwkv_gen.Q, layer, B, pos, 1, Hq, d, q[layer].data_ptr(), s)
+            hwkv_gen.fill_device(g, hwkv_gen.K, layer, B, pos, 1, Hkv, d, k[layer].data_ptr(), s)
+            hwkv_gen.fill_device(g, hwkv_gen.V, layer, B, pos, 1, Hkv, d, v[layer].data_ptr(), s)
+        return q, k, v
+
+    n_dev = args.warmup + args.steps
+    inputs = [gen_step(prompt + i) for i in range(n_dev)]
+    out = torch.empty((L, B, Hq, d), dtype=torch.float32, device=dev)
+    stream.synchronize()
+
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+            torch.cuda.Event(enable_timing=True)) for _ in range(L)] for _ in range(args.steps)]
+    resid = []
+
+    def step(i, timed_idx=None):
+        q, k, v = inputs[i]
+        for layer in range(L):
+            if timed_idx is not None:
+                ev[timed_idx][layer][0].record(stream)
+            hwkv.hwkv_append(cache, layer, k[layer], v[layer], 1, s)
+            if timed_idx is not None:
+                ev[timed_idx][layer][1].record(stream)
+            hwkv.hwkv_decode_attn(cache, layer, q[layer], scale, out[layer], s)
+            if timed_idx is not None:
+                ev[timed_idx][layer][2].record(stream)
+        resid.append(hwkv.hwkv_residency_bytes(cache, -1))
+
+    for i in range(args.warmup):
+        step(i)
+    t_first = hwkv.hwkv_seq_len(cache, 0)
+    stream.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for j in range(args.steps):
+            step(args.warmup + j, j)
+        end.record(stream)
+        end.synchronize()
+    torch.cuda.synchronize()
+    barrier(world)
+    ms_local = start.elapsed_time(end)
+    clocks = clk.summary()
+    hwkv.hwkv_sync_check(cache)
+
+    # decode launch durations and their algorithmic bytes
+    dec_ms, app_ms, dec_bytes = [], [], []
+    for j in range(args.steps):
+        t = t_first + j + 1
+        per_layer = decode_bytes(wl, max_ctx, t)
+        for layer in range(L):
+            e0, e1, e2 = ev[j][layer]
+            app_ms.append(e0.elapsed_time(e1))
+            dec_ms.append(e1.elapsed_time(e2))
+            dec_bytes.append(per_layer[layer])
+    dec_avg_ms = float(np.mean(dec_ms))
+    bytes_avg = float(np.mean(dec_bytes))
+    achieved_gbs = bytes_avg / (dec_avg_ms * 1e-3) / 1e9
+    step_bytes = float(np.sum(dec_bytes)) / args.steps
+
+    ms = max_over_ranks(ms_local, world)
+    tokens = sum_over_ranks(float(B * args.steps), world)
+    value = tokens / (ms * 1e-3)
+
+    # ---- end to end: host inputs in, host outputs out, every step
+    o_h = torch.empty((L, B, Hq, d), dtype=torch.float32, pin_memory=True)
+    q_d = torch.empty((L, B, Hq, d), dtype=torch.bfloat16, device=dev)
+    k_d = torch.empty((L, B, 1, Hkv, d), dtype=torch.bfloat16, device=dev)
+    v_d = torch.empty_like(k_d)
+    pos0 = hwkv.hwkv_seq_len(cache, 0)
+    host_inputs = []
+    for i in range(e2e_steps + 2):
+        q, k, v = gen_step(pos0 + i)
+        host_inputs.append((q.cpu().pin_memory(), k.cpu().pin_memory(), v.cpu().pin_memory()))
+    stream.synchronize()
+
+    def e2e_step(i):
+        qh, kh, vh = host_inputs[i]
+        q_d.copy_(qh, non_blocking=True)
+        k_d.copy_(kh, non_blocking=True)
+        v_d.copy_(vh, non_blocking=True)
+        for layer in range(L):
+            hwkv.hwkv_append(cache, layer, k_d[layer], v_d[layer], 1, s)
+            hwkv.hwkv_decode_attn(cache, layer, q_d[layer], scale, out[layer], s)
+        o_h.copy_(out, non_blocking=True)
+
+    for i in range(2):
+        e2e_step(i)
+    stream.synchronize()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_steps):
+        e2e_step(2 + i)
+    e1.record(stream)
+    e1.synchronize()
+    barrier(world)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+    e2e_value = sum_over_ranks(float(B * e2e_steps), world) / (e2e_ms * 1e-3)
+    h2d = int(sum(x.numel() * x.element_size() for x in host_inputs[0]))
+    d2h = int(o_h.numel() * 4)
+    t_end = hwkv.hwkv_seq_len(cache, 0)
+    resid_bytes = hwkv.hwkv_residency_bytes(cache, -1)
+    hwkv.hwkv_sync_check(cache)
+    hwkv.hwkv_free(cache)
+    del arena, inputs
+    torch.cuda.empty_cache()
+
+    return dict(value=value, ms=ms, e2e_value=e2e_value, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
+                dec_avg_ms=dec_avg_ms, app_avg_ms=float(np.mean(app_ms)), bytes_avg=bytes_avg,
+                achieved_gbs=achieved_gbs, step_bytes=step_bytes, clocks=clocks,
+                t_first=t_first, t_end=t_end, resid_bytes=resid_bytes,
+                launches=args.steps * L * 3, e2e_steps=e2e_steps, max_ctx=max_ctx)
+
+
+# ------------------------------------------------------------- GPU prefill
+def prefill_flops(wl, t0, n):
+    """Algorithmic flops of one prefill chunk: 4 d G per visible (query, key) pair."""
+    total = 0
+    for h in range(wl.n_kv_heads):
+        W = wl.windows[h]
+        # visible keys of query p: min(p + 1, W) (full: p + 1); sum over p in the chunk
+        if W == 0 or W >= wl.max_ctx:
+            pairs = sum_range(t0 + 1, t0 + n)
+        else:
+            lo, hi = t0 + 1, t0 + n  # p + 1 ranges over [lo, hi]
+            cut = min(max(W, lo - 1), hi)  # p + 1 <= W counts p + 1, above counts W
+            pairs = sum_range(lo, cut) + W * (hi - cut)
+        total += pairs * wl.group * 4 * wl.head_dim * wl.batch
+    return total
+
+
+def sum_range(a, b):
+    """a + (a+1) + ... + b (0 if b < a)."""
+    return 0 if b < a else (a + b) * (b - a + 1) // 2
+
+
+def run_prefill(args, local):
+    import torch
+
+    import hwkv_gen
+    import paper_2609_02029_gb300 as hwkv
+
+    wl = workloads.make("prefill64k")
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    s = stream.cuda_stream
+    g = hwkv_gen.desc(wl.seed, wl.per_head_scale)
+    B, Hq, Hkv, d, n = wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.chunk
+    chunks = wl.prompt // n
+    scale = 1.0 / np.sqrt(d)
+    q = torch.empty((chunks, B, n, Hq, d), dtype=torch.bfloat16, device=dev)
+    k = torch.empty((chunks, B, n, Hkv, d), dtype=torch.bfloat16, device=dev)
+    v = torch.empty_like(k)
+    for c in range(chunks):
+        hwkv_gen.fill_device(g, hwkv_gen.Q, 0, B, c * n, n, Hq, d, q[c].data_ptr(), s)
+        hwkv_gen.fill_device(g, hwkv_gen.K, 0, B, c * n, n, Hkv, d, k[c].data_ptr(), s)
+        hwkv_gen.fill_device(g, hwkv_gen.V, 0, B, c * n, n, Hkv, d, v[c].data_ptr(), s)
+    out = torch.empty((B, n, Hq, d), dtype=torch.float32, device=dev)
+    pol = hwkv.make_policy(1, Hkv, Hq, d, B, wl.max_ctx, wl.windows)
+    nbytes = hwkv.hwkv_required_bytes(pol)
+    arena = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    reps = []
+    flops = sum(prefill_flops(wl, c * n, n) for c in range(chunks))
+    for rep in range(1 + args.prefill_reps):
+        cache = hwkv.hwkv_alloc(pol, arena, nbytes, s)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for c in range(chunks):
+            hwkv.hwkv_prefill(cache, 0, q[c], k[c], v[c], n, scale, out, s)
+        e1.record(stream)
+        e1.synchronize()
+        hwkv.hwkv_sync_check(cache)
+        hwkv.hwkv_free(cache)
+        if rep > 0:
+            reps.append(e0.elapsed_time(e1))
+    ms = float(np.median(reps))
+    del q, k, v, out, arena
+    torch.cuda.empty_cache()
+    return dict(ms=ms, flops=flops, tflops=flops / (ms * 1e-3) / 1e12,
+                tokens_per_s=B * wl.prompt / (ms * 1e-3))
+
+
+# ------------------------------------------------------------ CPU oracle
+def step_keys(wl, max_ctx, t):
+    """(layer, batch row, KV head) units of one decode step at length t and the
+    keys each attends to."""
+    out = []
+    for l in range(wl.n_layers):
+        for h in range(wl.n_kv_heads):
+            W = wl.windows[l * wl.n_kv_heads + h]
+            cap = max_ctx if (W == 0 or W >= max_ctx) else W
+            for b in range(wl.batch):
+                out.append((l, b, h, W if cap == W else 0, min(t, cap)))
+    return out
+
+
+class OracleSample:
+    """A bounded sample of one decode step for the fp64 oracle (array form):
+    units drawn at random, their q/K/V generated on the host before any clock
+    starts, at most `max_bytes` of inputs held."""
+
+    def __init__(self, wl, max_ctx, t, max_units, max_bytes=3 << 30, seed=12345):
+        from concurrent.futures import ThreadPoolExecutor
+
+        import hwkv_gen
+        import oracle
+
+        self.wl, self.t = wl, t
+        self.cores = os.cpu_count() or 1
+        self.units_all = step_keys(wl, max_ctx, t)
+        self.keys_all = sum(u[4] for u in self.units_all)
+        g = hwkv_gen.desc(wl.seed, wl.per_head_scale)
+        d, G, p = wl.head_dim, wl.group, t - 1
+        rng = np.random.default_rng(seed)
+        order = rng.permutation(len(self.units_all))
+        chosen, held = [], 0
+        for i in order[:max_units]:
+            u = self.units_all[i]
+            nb = u[4] * d * 2 * 2
+            if chosen and held + nb > max_bytes:
+                break
+            chosen.append(u)
+            held += nb
+
+        def make(u):
+            l, b, h, W, n = u
+            lo = oracle.window_lo(p, W)
+            K = hwkv_gen.fill_host_sub(g, hwkv_gen.K, l, b, lo, p - lo + 1, h, 1, d)[:, 0]
+            V = hwkv_gen.fill_host_sub(g, hwkv_gen.V, l, b, lo, p - lo + 1, h, 1, d)[:, 0]
+            Q = hwkv_gen.fill_host_sub(g, hwkv_gen.Q, l, b, p, 1, h * G, G, d)[0]
+            return (Q, K, V, p - lo)
+
+        with ThreadPoolExecutor(max_workers=self.cores) as ex:
+            self.inputs = list(ex.map(make, chosen))
+        self.keys = [x[1].shape[0] for x in self.inputs]
+
+    def run(self, n_units=None):
+        """Seconds the oracle takes on the first n_units sampled units, all host
+        cores busy (one unit per thread, one OpenMP thread each)."""
+        import threading
+        from concurrent.futures import ThreadPoolExecutor
+
+        import oracle
+
+        units = self.inputs[:n_units] if n_units else self.inputs
+        local = threading.local()
+        d = self.wl.head_dim
+
+        def work(u):
+            if not getattr(local, "set", False):
+                oracle.set_threads(1)
+                local.set = True
+            Q, K, V, p_rel = u
+            oracle.window_attention_bf16(Q, [p_rel] * len(Q), K, V, 0, 1.0 / np.sqrt(d))
+
+        t0 = time.perf_counter()
+        with ThreadPoolExecutor(max_workers=self.cores) as ex:
+            list(ex.map(work, units))
+        return time.perf_counter() - t0, len(units), sum(self.keys[:len(units)])
+
+    def step_seconds(self, sec, keys):
+        """Whole-step time, scaling the sample by keys attended (cost is linear in keys)."""
+        return sec * self.keys_all / max(keys, 1)
+
+    def describe(self, n, keys, sec):
+        return ("%d of %d (layer, batch row, KV head) units of one decode step at t=%d, "
+                "%d of %d keys, fp64 oracle %.2f s on %d threads, scaled by keys to the full "
+                "step" % (n, len(self.units_all), self.t, keys, self.keys_all, sec, self.cores))
+
+
+def cpu_baseline(wl, max_ctx, t, budget_s=15.0):
+    """Oracle tokens/s on this host's cores from a bounded sample of one step."""
+    cores = os.cpu_count() or 1
+    samp = OracleSample(wl, max_ctx, t, max_units=8 * cores)
+    sec, n, keys = samp.run()
+    if sec > budget_s and n > cores:  # keep the timed work bounded
+        m = max(cores, int(n * budget_s / sec))
+        sec, n, keys = samp.run(m)
+    step_s = samp.step_seconds(sec, keys)
+    return {"value": wl.batch / step_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": samp.describe(n, keys, sec)}
+
+
+# ------------------------------------------------------------------ main
+def emit(obj):
+    print(json.dumps(obj), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=96)
+    ap.add_argument("--warmup", type=int, default=4)
+    ap.add_argument("--workload", default="layers16_112k",
+                    choices=["layers16_112k", "single32k", "budget161k_r25", "budget161k_r50",
+                             "budget161k_r75", "budget161k_r100"])
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=32)
+    ap.add_argument("--prefill-reps", type=int, default=3)
+    ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling only: keep the first N layers (the reported workload is "
+                         "the full one)")
+    ap.add_argument("--batch", type=int, default=0, help="profiling only: batch rows")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    if args.workload.startswith("budget161k_r"):
+        wl = workloads.make("budget161k", int(args.workload.split("_r")[1]) / 100.0)
+    else:
+        wl = workloads.make(args.workload)
+    if args.layers:
+        wl.n_layers = args.layers
+        wl.windows = wl.windows[:args.layers * wl.n_kv_heads]
+        wl.name += "_L%d" % args.layers
+    if args.batch:
+        wl.batch = args.batch
+        wl.name += "_B%d" % args.batch
+    hbm, tf_burst, tf_sust, peak_src = peaks()
+    world, rank, local = dist_setup(args.gpus)
+    metric = "decode attn tokens/s on per-head-window KV"
+    config = {"workload": wl.name, "layers": wl.n_layers, "batch_per_gpu": wl.batch,
+              "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
+              "context": wl.max_ctx, "window_levels": wl.levels, "note": wl.note,
+              "parallelism": "replicas" if args.gpus > 1 else "single",
+              "l2": "inputs larger than L2 (each layer-step reads > 129 MB of K/V)"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        max_ctx = wl.max_ctx
+        t = wl.prompt + 1
+        cores = os.cpu_count() or 1
+        samp = OracleSample(wl, max_ctx, t, max_units=4 * cores)
+        budget = max(0.5, 120.0 / (args.steps + args.warmup))  # whole run within minutes
+        sec, n, keys = samp.run()
+        m = n if sec <= budget else max(1, int(n * budget / sec))
+        times = []
+        for i in range(args.warmup + args.steps):
+            sec, n, keys = samp.run(m)
+            if i >= args.warmup:
+                times.append(samp.step_seconds(sec, keys))
+        step_s = float(np.mean(times))
+        v = wl.batch / step_s
+        emit({"metric": metric, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
+              "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+              "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+              "data": "synthetic", "config": config, "impl": "reference",
+              "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                               "sample": samp.describe(n, keys, sec) + "; each step"},
+              "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                      "d2h_bytes_per_step": 0}})
+        return
+
+    r = run_gpu(args, wl, world, rank, local)
+    pre = None
+    if not args.no_prefill and rank == 0:
+        pre = run_prefill(args, local)
+    cb = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cb = cpu_baseline(wl, r["max_ctx"], r["t_first"] + 1)
+    if rank != 0:
+        return
+    config["context"] = r["t_end"]
+    line = {
+        "metric": metric, "value": r["value"], "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["ms"] / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic", "config": config,
+        "hbm_gbs": r["step_bytes"] / (r["ms"] / args.steps * 1e-3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": "hwkv_decode_attn (split kernel + combine)",
+                     "achieved": r["achieved_gbs"], "peak": hbm, "unit": "GB/s",
+                     "frac": r["achieved_gbs"] / hbm, "peak_source": peak_src,
+                     "frac_of_nominal_8tbs": r["achieved_gbs"] / NOMINAL_HBM_GBS,
+                     "bytes_per_launch": r["bytes_avg"], "launch_ms": r["dec_avg_ms"],
+                     "traffic": None},
+        "append_ms_per_launch": r["app_avg_ms"],
+        "residency_bytes": r["resid_bytes"],
+        "e2e": {"value": r["e2e_value"], "unit": "tokens/s", "h2d_bytes_per_step": r["h2d"],
+                "d2h_bytes_per_step": r["d2h"], "steps": r["e2e_steps"]},
+        "gpu_launches": r["launches"],
+        "clocks": r["clocks"],
+    }
+    if pre is not None:
+        line["prefill"] = {"workload": "prefill64k", "tflops": pre["tflops"],
+                           "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst,
+                           "peak_source": peak_src, "ms": pre["ms"],
+                           "tokens_per_s": pre["tokens_per_s"], "flops": pre["flops"]}
+    if cb is not None:
+        line["cpu_baseline"] = cb
+    emit(line)
+
+
+if __name__ == "__main__":
+    main()

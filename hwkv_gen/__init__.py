@@ -38,6 +38,11 @@ def _host_lib():
                                            ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                            ctypes.c_void_p]
         lib.hwkv_gen_fill_host.restype = ctypes.c_int
+        lib.hwkv_gen_fill_host_sub.argtypes = [
+            ctypes.POINTER(GenDesc), ctypes.c_uint32, ctypes.c_uint32, ctypes.c_int32,
+            ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_int32, ctypes.c_void_p]
+        lib.hwkv_gen_fill_host_sub.restype = ctypes.c_int
         lib.hwkv_gen_one.argtypes = [ctypes.POINTER(GenDesc), ctypes.c_uint32, ctypes.c_uint32,
                                      ctypes.c_uint32, ctypes.c_uint32, ctypes.c_int64,
                                      ctypes.c_uint32]
@@ -73,6 +78,16 @@ def fill_host(g, tensor, layer, B, pos0, n, H, d):
     if rc != 0:
         raise ValueError("hwkv_gen_fill_host: bad arguments")
     return out
+
+
+def fill_host_sub(g, tensor, layer, b, pos0, n, head0, H, d):
+    """uint16 array [n, H, d]: batch row b and heads head0 .. head0+H-1 only."""
+    out = np.empty((1, n, H, d), dtype=np.uint16)
+    rc = _host_lib().hwkv_gen_fill_host_sub(ctypes.byref(g), tensor, layer, b, 1, pos0, n, head0,
+                                            H, d, out.ctypes.data_as(ctypes.c_void_p))
+    if rc != 0:
+        raise ValueError("hwkv_gen_fill_host_sub: bad arguments")
+    return out[0]
 
 
 def one(g, tensor, layer, b, head, pos, dim):

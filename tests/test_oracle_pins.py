@@ -294,3 +294,10 @@ def test_generator_distribution_and_scale():
     for h in range(4):
         s = hwkv_gen.head_scale(gs, hwkv_gen.K, 3, h)
         assert abs(y[0, :, h].std() / s - 1) < 0.03
+
+
+def test_generator_sub_fill_matches_full_fill():
+    g = hwkv_gen.desc(seed=4, per_head_scale=True)
+    full = hwkv_gen.fill_host(g, hwkv_gen.V, 2, 3, 10, 20, 5, 16)
+    sub = hwkv_gen.fill_host_sub(g, hwkv_gen.V, 2, 2, 10, 20, 1, 3, 16)
+    assert np.array_equal(sub, full[2, :, 1:4])
