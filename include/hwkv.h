@@ -146,6 +146,32 @@ HWKV_API hwkv_status hwkv_prefill(hwkv_cache* cache, int32_t layer, const void* 
 HWKV_API hwkv_status hwkv_decode_attn(hwkv_cache* cache, int32_t layer, const void* q, float scale,
                              float* out, void* cuda_stream);
 
+/* Size of the device array hwkv_decode_attn_static keeps its scratch in. */
+#define HWKV_DECODE_STATIC_SCRATCH_BYTES (4u << 20)
+
+/*
+ * The paper has no counterpart of this call; it serves callers that cannot
+ * allocate device memory. Plugins running inside another engine whose
+ * allocator owns all GPU memory, code that must never synchronize the device
+ * (cudaMalloc and cudaFree can), and code issued during stream capture are
+ * handed their inputs and outputs but cannot create scratch buffers.
+ *
+ * Same result and arguments as hwkv_decode_attn, but the per-tile partials
+ * live in a fixed 4 MiB array inside this library's device image (present on
+ * every GPU that loads the library until the process exits) instead of the
+ * cache's workspace. It calls no cudaMalloc, cudaFree or allocating routine.
+ * The first call on each device, with that device current, looks up the
+ * array's device address (cudaGetSymbolAddress); make that first call before
+ * any stream capture. The array keeps the last call's contents and nothing in
+ * it needs to start at zero. All calls share it: calls whose kernels overlap
+ * on the GPU (other streams, other caches) race and give wrong results.
+ * Fails with HWKV_EINVAL when batch * n_kv_heads exceeds the tiles the array
+ * holds ((4 MiB - 256) / (32 * head_dim + 64): 508 at head_dim 256, 1008
+ * at 128, 1985 at 64), before anything is launched.
+ */
+HWKV_API hwkv_status hwkv_decode_attn_static(hwkv_cache* cache, int32_t layer, const void* q,
+                                             float scale, float* out, void* cuda_stream);
+
 /*
  * Resident K+V bytes (Sec. 3.1, Eq. nominal-storage with C = t, bf16 K and V,
  * times batch): sum over KV heads of batch * min(cap, t) * head_dim * 2 * 2,

@@ -11,6 +11,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -318,7 +319,8 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
 // Decode tile plan: equal-length tiles (multiple of 64 tokens) over every
 // (batch row, KV head) ring. The length is chosen to balance the persistent
 // grid: minimise (tiles per CTA) x (tile length + a fixed per-tile cost).
-static void plan_decode(const hwkv_cache* c, int32_t layer, DecodeParams& p, int& grid) {
+static void plan_decode(const hwkv_cache* c, int32_t layer, int max_tiles, DecodeParams& p,
+                        int& grid) {
   const int H = c->pol.n_kv_heads, B = c->pol.batch;
   const int64_t t = c->t[layer];
   int64_t n_valid[kMaxKvHeads];
@@ -341,7 +343,7 @@ static void plan_decode(const hwkv_cache* c, int32_t layer, DecodeParams& p, int
   for (int64_t len = 128; ; len = len < 1024 ? len + 64 : len + len / 8 / 64 * 64) {
     const int64_t L = std::min(len, max_len);
     const int64_t nt = count(L);
-    if (nt <= c->lay.max_tiles) {
+    if (nt <= max_tiles) {
       const int64_t g = std::min<int64_t>(nt, sms);
       const double cost = (double)((nt + g - 1) / g) * (double)(L + per_tile_cost);
       if (best_len == 0 || cost < best) {
@@ -390,7 +392,7 @@ hwkv_status hwkv_decode_attn(hwkv_cache* c, int32_t layer, const void* q, float 
   p.out = out;
   p.err = c->err();
   int grid = 0;
-  plan_decode(c, layer, p, grid);
+  plan_decode(c, layer, c->lay.max_tiles, p, grid);
   if (p.n_tiles > c->lay.max_tiles)
     return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
@@ -479,6 +481,94 @@ hwkv_status hwkv_sync_check(hwkv_cache* c) {
     return fail(HWKV_EKERNEL, "kernel error word 0x%x (1 = bounded wait gave up, 2 = bad index)",
                 word);
   }
+  return ok();
+}
+
+// ---------------------------------------------------------------------------
+// Decode without any device allocation. Some callers cannot allocate device
+// memory at all: code embedded in another engine whose allocator owns every
+// byte of the GPU, code that must never synchronize the device (cudaMalloc and
+// cudaFree can), and code issued while a stream is being captured. They own
+// the cache arena and the q/out tensors, but cannot provide scratch. This
+// entry point keeps the decode tile partials in a fixed array that lives in
+// the library's own device image instead of the cache's workspace.
+//
+// The array is HWKV_DECODE_STATIC_SCRATCH_BYTES (4 MiB) on every GPU that
+// loads this library, held until the process exits. Host code cannot use the
+// array's name as a device address (on the host it is only a stand-in), so
+// the first call on each device, with that device current, looks the address
+// up with cudaGetSymbolAddress and keeps it; that first call should come
+// before any stream capture. Every call shares the array and it keeps the
+// last call's contents; nothing in it has to start at zero (each tile partial
+// is written before it is read). Calls whose kernels overlap on the GPU (two
+// streams, or two caches, at once) race on it.
+static __device__ __align__(256) uint8_t g_decode_static_scratch[HWKV_DECODE_STATIC_SCRATCH_BYTES];
+
+static void* static_scratch_address(int device, cudaError_t* err) {
+  constexpr int kMaxDevices = 64;
+  static std::mutex mu;
+  static void* addr[kMaxDevices] = {};
+  std::lock_guard<std::mutex> lock(mu);
+  *err = cudaSuccess;
+  if (device < 0 || device >= kMaxDevices) {
+    *err = cudaErrorInvalidDevice;
+    return nullptr;
+  }
+  if (!addr[device]) {
+    void* ptr = nullptr;
+    *err = cudaGetSymbolAddress(&ptr, g_decode_static_scratch);
+    if (*err != cudaSuccess) return nullptr;
+    addr[device] = ptr;
+  }
+  return addr[device];
+}
+
+hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q, float scale,
+                                    float* out, void* cuda_stream) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (!q || !out) return fail(HWKV_EINVAL, "q/out is NULL");
+  if (c->t[layer] <= 0) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
+  if (c->t[layer] > INT32_MAX) return fail(HWKV_EUNSUPPORTED, "ring longer than 2^31");
+  const int d = c->pol.head_dim;
+  const size_t o_bytes_per_tile = (size_t)kMaxGroup * d * 4;
+  const size_t ml_bytes_per_tile = (size_t)kMaxGroup * 8;
+  const int cap_tiles =
+      (int)((HWKV_DECODE_STATIC_SCRATCH_BYTES - kAlign) / (o_bytes_per_tile + ml_bytes_per_tile));
+  const int min_tiles = c->pol.batch * c->pol.n_kv_heads;  // one tile per (batch row, KV head)
+  if (min_tiles > cap_tiles)
+    return fail(HWKV_EINVAL,
+                "batch x n_kv_heads = %d exceeds the %d tiles the %d-byte static decode scratch "
+                "holds at head_dim %d",
+                min_tiles, cap_tiles, (int)HWKV_DECODE_STATIC_SCRATCH_BYTES, d);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+  uint8_t* scratch = static_cast<uint8_t*>(static_scratch_address(dev, &e));
+  if (!scratch)
+    return fail(HWKV_ECUDA, "cudaGetSymbolAddress(static decode scratch) on device %d: %s", dev,
+                cudaGetErrorString(e));
+  DecodeParams p{};
+  p.n_units = c->pol.n_kv_heads;
+  p.batch = c->pol.batch;
+  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
+  p.n_q_heads = c->pol.n_q_heads;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.part_o = reinterpret_cast<float*>(scratch);
+  p.part_ml = reinterpret_cast<float2*>(scratch + align_up((size_t)cap_tiles * o_bytes_per_tile, kAlign));
+  p.out = out;
+  p.err = c->err();
+  int grid = 0;
+  plan_decode(c, layer, cap_tiles, p, grid);
+  if (p.n_tiles > cap_tiles)
+    return fail(HWKV_EINVAL, "decode plan needs %d tiles > %d in the static scratch", p.n_tiles,
+                cap_tiles);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  e = launch_decode(p, c->kv_map, d, grid, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
+  e = launch_decode_combine(p, d, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
   return ok();
 }
 
