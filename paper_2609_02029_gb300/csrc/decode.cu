@@ -274,7 +274,11 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     }
     consumer_sync();
     {
+      // one tile covers the whole ring: this is the final output, normalised here;
+      // otherwise leave the tile's partial for the combine kernel
+      const bool single = p.u[ti.h].n_tiles == 1;
       float* po = p.part_o + (int64_t)tile * kMaxGroup * D;
+      float* fo = p.out + ((int64_t)ti.b * p.n_q_heads + (int64_t)ti.h * p.group) * D;
       for (int n = 0; n < p.group; ++n) {
         float M = -INFINITY;
 #pragma unroll
@@ -286,44 +290,95 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
           e[ww] = ml.x == -INFINITY ? 0.f : ex2((ml.x - M) * c);
           L += e[ww] * ml.y;
         }
+        const float scale_out = single ? 1.f / L : 1.f;
+        float* dst = single ? fo + (int64_t)n * D : po + (int64_t)n * D;
         for (int i = w * (D / kDecodeWarps) + lane; i < (w + 1) * (D / kDecodeWarps); i += 32) {
           float acc = 0.f;
 #pragma unroll
           for (int ww = 0; ww < kDecodeWarps; ++ww)
             acc += e[ww] * red_o[((size_t)ww * kMaxGroup + n) * C::kRedLd + i];
-          po[(int64_t)n * D + i] = acc;
+          dst[i] = acc * scale_out;
         }
-        if (w == 0 && lane == 0) p.part_ml[(int64_t)tile * kMaxGroup + n] = make_float2(M, L);
+        if (!single && w == 0 && lane == 0)
+          p.part_ml[(int64_t)tile * kMaxGroup + n] = make_float2(M, L);
       }
     }
   }
 }
 
-// Log-sum-exp merge of the tile partials of one (batch row, KV head):
-// o = sum_i 2^{(m_i - M) c} o_i / sum_i 2^{(m_i - M) c} l_i, M = max_i m_i,
-// over the tiles in their fixed order (deterministic).
+// Log-sum-exp merge of the tile partials of one (batch row, query head):
+// o = sum_j 2^{(m_j - M) c} o_j / sum_j 2^{(m_j - M) c} l_j, M = max_j m_j,
+// over the head's tiles in their fixed order (deterministic). One CTA per
+// (batch row, query head, 128-channel chunk); the tile weights are computed
+// once into shared memory, then each thread sums its channel over the tiles.
+// Heads whose ring is a single tile were written by the split kernel.
 template <int D>
-__global__ void __launch_bounds__(D) decode_combine_kernel(const DecodeParams p) {
-  const int b = blockIdx.x / p.n_units;
-  const int h = blockIdx.x - b * p.n_units;
-  const int i = threadIdx.x;
+__global__ void __launch_bounds__(D < 128 ? D : 128) decode_combine_kernel(const DecodeParams p) {
+  constexpr int NT = D < 128 ? D : 128;
+  constexpr int CH = D / NT;
+  __shared__ float s_w[kCombineMaxTiles];
+  __shared__ float s_red[NT / 32];
+  __shared__ float s_bcast;
+  const int chunk = blockIdx.x % CH;
+  const int bq = blockIdx.x / CH;
+  const int b = bq / p.n_q_heads;
+  const int qh = bq - b * p.n_q_heads;
+  const int h = qh / p.group;
+  const int n = qh - h * p.group;
   const DecodeUnit& u = p.u[h];
-  const int64_t tile0 = (int64_t)b * p.tiles_per_b + u.tile_begin;
   const int n_t = u.n_tiles;
+  if (n_t <= 1) return;
+  const int64_t tile0 = (int64_t)b * p.tiles_per_b + u.tile_begin;
   const float c = p.scale_log2;
-  for (int n = 0; n < p.group; ++n) {
-    float M = -INFINITY;
-    for (int j = 0; j < n_t; ++j) M = fmaxf(M, p.part_ml[(tile0 + j) * kMaxGroup + n].x);
-    float num = 0.f, den = 0.f;
-    for (int j = 0; j < n_t; ++j) {
-      const float2 ml = p.part_ml[(tile0 + j) * kMaxGroup + n];
-      if (ml.x == -INFINITY) continue;
-      const float wgt = ex2((ml.x - M) * c);
-      num += wgt * p.part_o[((tile0 + j) * kMaxGroup + n) * D + i];
-      den += wgt * ml.y;
-    }
-    p.out[((int64_t)b * p.n_q_heads + (int64_t)h * p.group + n) * D + i] = num / den;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+
+  // M = max_j m_j
+  float mx = -INFINITY;
+  for (int j = tid; j < n_t; j += NT) mx = fmaxf(mx, p.part_ml[(tile0 + j) * kMaxGroup + n].x);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  if (lane == 0) s_red[wid] = mx;
+  __syncthreads();
+  if (tid == 0) {
+    float m = s_red[0];
+    for (int k = 1; k < NT / 32; ++k) m = fmaxf(m, s_red[k]);
+    s_bcast = m;
   }
+  __syncthreads();
+  const float M = s_bcast;
+  // weights and L = sum_j w_j l_j
+  float lsum = 0.f;
+  for (int j = tid; j < n_t; j += NT) {
+    const float2 ml = p.part_ml[(tile0 + j) * kMaxGroup + n];
+    const float wj = ml.x == -INFINITY ? 0.f : ex2((ml.x - M) * c);
+    s_w[j] = wj;
+    lsum += wj * ml.y;
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+  __syncthreads();
+  if (lane == 0) s_red[wid] = lsum;
+  __syncthreads();
+  if (tid == 0) {
+    float l = 0.f;
+    for (int k = 0; k < NT / 32; ++k) l += s_red[k];
+    s_bcast = l;
+  }
+  __syncthreads();
+  const float L = s_bcast;
+  const int i = chunk * NT + tid;
+  const float* src = p.part_o + (tile0 * kMaxGroup + n) * D + i;
+  const int64_t stride = (int64_t)kMaxGroup * D;
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  int j = 0;
+  for (; j + 4 <= n_t; j += 4) {
+    a0 += s_w[j] * src[(j + 0) * stride];
+    a1 += s_w[j + 1] * src[(j + 1) * stride];
+    a2 += s_w[j + 2] * src[(j + 2) * stride];
+    a3 += s_w[j + 3] * src[(j + 3) * stride];
+  }
+  for (; j < n_t; ++j) a0 += s_w[j] * src[j * stride];
+  p.out[((int64_t)b * p.n_q_heads + qh) * D + i] = ((a0 + a1) + (a2 + a3)) / L;
 }
 
 int decode_smem_bytes(int head_dim) {
@@ -357,11 +412,14 @@ cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& map, int hea
 }
 
 cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s) {
-  const int grid = p.batch * p.n_units;
+  bool any = false;  // nothing to merge when every ring is a single tile
+  for (int h = 0; h < p.n_units; ++h) any |= p.u[h].n_tiles > 1;
+  if (!any) return cudaSuccess;
+  const int bq = p.batch * p.n_q_heads;
   switch (head_dim) {
-    case 64: decode_combine_kernel<64><<<grid, 64, 0, s>>>(p); break;
-    case 128: decode_combine_kernel<128><<<grid, 128, 0, s>>>(p); break;
-    case 256: decode_combine_kernel<256><<<grid, 256, 0, s>>>(p); break;
+    case 64: decode_combine_kernel<64><<<bq, 64, 0, s>>>(p); break;
+    case 128: decode_combine_kernel<128><<<bq, 128, 0, s>>>(p); break;
+    case 256: decode_combine_kernel<256><<<bq * 2, 128, 0, s>>>(p); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

@@ -16,6 +16,7 @@ constexpr int kMaxKvHeads = 64;
 constexpr int kMaxGroup = 8;          // query heads per KV head handled by one mma n-tile
 constexpr int kDecodeWarps = 4;       // consumer warps per decode CTA
 constexpr int kStageTokens = 64;      // tokens per pipeline stage (16 per consumer warp)
+constexpr int kCombineMaxTiles = 4096;  // tiles of one ring the combine kernel can merge
 constexpr int kSlabBytes = 64 * 128;  // one TMA box: 64 rows x 128 B (64 bf16)
 
 // error word bits (set with atomicOr, read by hwkv_sync_check)
@@ -43,8 +44,8 @@ struct DecodeParams {
   int32_t n_tiles;      // batch * tiles_per_b
   float scale_log2;     // scale * log2(e)
   const __nv_bfloat16* q;  // [batch][n_q_heads][D]
-  float* part_o;           // [n_tiles * kDecodeWarps][D][kMaxGroup]
-  float2* part_ml;         // [n_tiles * kDecodeWarps][kMaxGroup]  (max, sum)
+  float* part_o;           // [n_tiles][kMaxGroup][D]: unnormalised tile outputs
+  float2* part_ml;         // [n_tiles][kMaxGroup]: (max logit, sum of weights)
   float* out;              // [batch][n_q_heads][D]
   int* err;
   DecodeUnit u[kMaxKvHeads];

@@ -370,6 +370,7 @@ static void plan_decode(const hwkv_cache* c, int32_t layer, int max_tiles, Decod
   }
   p.tiles_per_b = begin;
   p.n_tiles = begin * B;
+  // per-ring tiles are bounded by max_tiles / batch <= max(2048, 2 * n_kv_heads) < kCombineMaxTiles
   grid = std::min(p.n_tiles, sms);
 }
 
