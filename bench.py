@@ -507,6 +507,8 @@ def main():
     ap.add_argument("--prefill-reps", type=int, default=3)
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--prefill-only", action="store_true",
+                    help="run only the 64K prefill measurement (profiling)")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: keep the first N layers (the reported workload is "
                          "the full one)")
@@ -562,6 +564,13 @@ def main():
                       "d2h_bytes_per_step": 0}})
         return
 
+    if args.prefill_only:
+        pre = run_prefill(args, local)
+        emit({"metric": "prefill TFLOP/s", "value": pre["tflops"], "unit": "TFLOP/s",
+              "n_gpus": 1, "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+              "config": {"workload": "prefill64k"}, "ms": pre["ms"], "flops": pre["flops"],
+              "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst, "peak_source": peak_src})
+        return
     r = run_gpu(args, wl, world, rank, local)
     pre = None
     if not args.no_prefill and rank == 0:

@@ -1,0 +1,507 @@
+// prefill_tc.cu -- window-limited causal prefill on the 5th-generation tensor
+// cores (tcgen05 + TMEM + TMA) (HeadWiseKV Sec. 3.2, Eq. conditional-attention-
+// weight and Eq. conditional-attention for every prompt position; Sec. 3.3:
+// each KV head reads only its own ring).
+//
+// Query p in [t0, t0+n) of query head q attends to KV head q/G at positions
+// [max(0, p-W+1), p]: positions < t0 from the head's ring, >= t0 from the
+// chunk's own K/V. The ring is walked in slot order (slot j holds the unique
+// retained position congruent to j mod cap), so wrap needs no special case;
+// each key column carries its position and the window/causal mask is applied
+// per element on the tiles that need it. Tiles no row of the block can see are
+// never loaded, so a short-window head does window-sized work.
+//
+// CTA = one 128-row query tile: 128/G positions x the G query heads of one KV
+// head (the GQA group shares every K/V tile). Warp roles:
+//   warp 0      TMA producer: Q once, then K/V tiles into a STAGES-deep ring
+//   warp 1      MMA issuer (one thread): S = Q K^T into a double-buffered TMEM
+//               tile (128 x BN fp32), then O += P V into TMEM (128 x D fp32)
+//   warps 2-5   softmax: thread r owns TMEM lane r = query row r, so the row
+//               max and sum are thread-local; P goes to shared memory as bf16
+//               (128-byte swizzle) for the PV mma; O is rescaled in TMEM only
+//               when a row's running max grows by more than 2^8 (the final
+//               O / l uses the same reference, so the result is exact).
+// While the softmax warps work on tile j the tensor core computes S of tile j+1.
+// All waits are bounded; a thread that gives up stops waiting and issuing but
+// keeps walking the tile sequence, so every role reaches the TMEM release.
+#include "hwkv_internal.cuh"
+
+namespace hwkv {
+
+namespace {
+
+template <int D, int BN, int STAGES>
+struct TcCfg {
+  static constexpr int kSlabs = D / 64;
+  static constexpr int kQSlab = 128 * 128;             // 128 rows x 128 B
+  static constexpr int kQBytes = kSlabs * kQSlab;
+  static constexpr int kKVSlab = BN * 128;             // BN rows x 128 B
+  static constexpr int kTileBytes = kSlabs * kKVSlab;  // one K (or V) tile
+  static constexpr int kStageBytes = 2 * kTileBytes;
+  static constexpr int kPSlab = 128 * 128;             // P: 128 rows x 64 keys
+  static constexpr int kPBytes = (BN / 64) * kPSlab;  // one P buffer; two are kept
+  static constexpr int kBarBytes = 256;
+  static constexpr int kSmem = kQBytes + STAGES * kStageBytes + 2 * kPBytes + kBarBytes + 1024;
+  static constexpr uint32_t kTmemCols = 512;
+  static_assert(2 * BN + D <= 512, "TMEM: two S buffers and O");
+};
+
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int32_t x,
+                                            int32_t y, int32_t z, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// The key tiles one query block needs, in order: ring slot tiles whose newest
+// held position reaches the block's lowest visible key, then chunk tiles up to
+// the block's last row. Every role walks the same sequence.
+template <int BN>
+struct KeySeq {
+  int64_t t0, n, W, cap, n_hist, r0, lo_need, c_first, n_chunk_tiles, n_hist_tiles;
+  bool hist_needed;
+  int64_t hist_cur, chunk_cur;
+
+  __device__ void init(const PrefillUnit& u, int64_t t0_, int64_t n_, int64_t p0, int64_t p_last) {
+    t0 = t0_;
+    n = n_;
+    W = u.window;
+    cap = u.cap;
+    n_hist = t0 < cap ? t0 : cap;
+    r0 = t0 % cap;
+    lo_need = W == 0 ? 0 : (p0 - W + 1 > 0 ? p0 - W + 1 : 0);
+    n_hist_tiles = (n_hist + BN - 1) / BN;
+    const int64_t c_lo = (t0 > lo_need ? t0 : lo_need) - t0;
+    c_first = (c_lo / BN) * BN;
+    const int64_t c_hi = p_last - t0;
+    n_chunk_tiles = c_hi >= c_first ? (c_hi - c_first) / BN + 1 : 0;
+    hist_needed = n_hist > 0 && (W == 0 || p0 - W + 1 < t0);
+    hist_cur = next_hist(0);
+    chunk_cur = 0;
+  }
+  __device__ int64_t slot_pos(int64_t j) const {
+    if (t0 <= cap) return j;
+    return j < r0 ? t0 - r0 + j : t0 - r0 - cap + j;
+  }
+  // smallest and largest position held in ring slots [j0, j1] (j1 < n_hist)
+  __device__ int64_t tile_min_pos(int64_t j0, int64_t j1) const {
+    if (t0 > cap && j0 < r0 && r0 <= j1) return slot_pos(r0);
+    return slot_pos(j0);
+  }
+  __device__ int64_t tile_max_pos(int64_t j0, int64_t j1) const {
+    if (t0 > cap && j0 < r0 && r0 <= j1) return slot_pos(r0 - 1);
+    return slot_pos(j1);
+  }
+  __device__ bool ring_tile_needed(int64_t jt) const {
+    if (!hist_needed) return false;
+    if (W == 0) return true;
+    const int64_t j0 = jt * BN;
+    const int64_t j1 = (j0 + BN < n_hist ? j0 + BN : n_hist) - 1;
+    return tile_max_pos(j0, j1) >= lo_need;
+  }
+  __device__ int64_t next_hist(int64_t jt) const {
+    for (; jt < n_hist_tiles; ++jt)
+      if (ring_tile_needed(jt)) return jt;
+    return -1;
+  }
+  __device__ bool next(int& hist, int64_t& j0) {
+    if (hist_cur >= 0) {
+      hist = 1;
+      j0 = hist_cur * BN;
+      hist_cur = next_hist(hist_cur + 1);
+      return true;
+    }
+    if (chunk_cur < n_chunk_tiles) {
+      hist = 0;
+      j0 = c_first + chunk_cur * BN;
+      ++chunk_cur;
+      return true;
+    }
+    return false;
+  }
+};
+
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, int* err,
+                                              bool& aborted) {
+  if (aborted) return false;
+  if (!mbar_wait_sleep_bounded(bar, parity, err)) aborted = true;
+  return !aborted;
+}
+
+// one lane of the warp waits, the warp then proceeds together; the abort flag
+// is shared by the warp so every lane takes the same path
+__device__ __forceinline__ bool warp_wait_or_abort(uint64_t* bar, uint32_t parity, int* err,
+                                                   bool& aborted) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = wait_or_abort(bar, parity, err, aborted) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  aborted = ok == 0;
+  return ok != 0;
+}
+
+}  // namespace
+
+template <int D, int BN, int STAGES>
+__global__ void __launch_bounds__(192, 1)
+    prefill_tc_kernel(const __grid_constant__ CUtensorMap q_map,
+                      const __grid_constant__ CUtensorMap ck_map,
+                      const __grid_constant__ CUtensorMap cv_map,
+                      const __grid_constant__ CUtensorMap ring_map, const PrefillParams p) {
+  using C = TcCfg<D, BN, STAGES>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sStage = smem + C::kQBytes;
+  uint8_t* sP = sStage + STAGES * C::kStageBytes;  // [2] P buffers
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * C::kPBytes);
+  uint64_t* kv_full = bars;              // [STAGES] TMA landed
+  uint64_t* kv_empty = bars + STAGES;    // [STAGES] PV of that tile done
+  uint64_t* s_full = bars + 2 * STAGES;  // [2] S tile computed
+  uint64_t* s_free = s_full + 2;         // [2] S tile read by the softmax warps
+  uint64_t* p_full = s_free + 2;         // [2] P buffer written (and O rescaled)
+  uint64_t* pv_done = p_full + 2;        // [2] PV mma that read that P buffer done
+  uint64_t* q_full = pv_done + 2;
+  uint64_t* o_full = q_full + 1;
+  uint64_t* drain = o_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = p.group;
+  const int QP = 128 / G;           // query positions per tile
+  const int rows_valid = QP * G;    // rows that carry a (position, head)
+  const int n_qblocks = (int)((p.n + QP - 1) / QP);
+  const int qb = n_qblocks - 1 - (int)blockIdx.x;  // longest rows first
+  const int h = blockIdx.y;
+  const int b = blockIdx.z;
+  const PrefillUnit& u = p.u[h];
+  const int64_t t0 = p.t0;
+  const int64_t p0 = t0 + (int64_t)qb * QP;
+  const int64_t p_last = min(p0 + QP, t0 + p.n) - 1;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_free[i], 4);  // one arrival per softmax warp
+      mbar_init(&p_full[i], 4);
+      mbar_init(&pv_done[i], 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(o_full, 1);
+    mbar_init(drain, 1);
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tmem_slot, C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  KeySeq<BN> seq;
+  seq.init(u, t0, p.n, p0, p_last);
+  bool aborted = false;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      prefetch_tensormap(&q_map);
+      prefetch_tensormap(&ck_map);
+      prefetch_tensormap(&cv_map);
+      prefetch_tensormap(&ring_map);
+      mbar_arrive_expect_tx(q_full, (uint32_t)(C::kSlabs * rows_valid * 128));
+      const int32_t qrow = (int32_t)((int64_t)b * p.n + (int64_t)qb * QP);
+#pragma unroll
+      for (int sl = 0; sl < C::kSlabs; ++sl)
+        tma_load_3d(sQ + sl * C::kQSlab, &q_map, sl * 64, h * G, qrow, q_full);
+      const int64_t krow0 = u.k_row0 + (int64_t)b * u.cap;
+      const int64_t vrow0 = u.v_row0 + (int64_t)b * u.cap;
+      uint32_t it = 0;
+      int hist;
+      int64_t j0;
+      while (seq.next(hist, j0)) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1u;
+        if (wait_or_abort(&kv_empty[s], ph ^ 1u, p.err, aborted)) {
+          uint8_t* kd = sStage + s * C::kStageBytes;
+          uint8_t* vd = kd + C::kTileBytes;
+          mbar_arrive_expect_tx(&kv_full[s], C::kStageBytes);
+#pragma unroll
+          for (int sl = 0; sl < C::kSlabs; ++sl) {
+#pragma unroll
+            for (int hf = 0; hf < BN / 64; ++hf) {
+              const uint32_t off = sl * C::kKVSlab + hf * 64 * 128;
+              if (hist) {
+                tma_load_2d(kd + off, &ring_map, sl * 64, (int32_t)(krow0 + j0 + hf * 64), &kv_full[s]);
+                tma_load_2d(vd + off, &ring_map, sl * 64, (int32_t)(vrow0 + j0 + hf * 64), &kv_full[s]);
+              } else {
+                const int32_t z = (int32_t)((int64_t)b * p.n + j0 + hf * 64);
+                tma_load_3d(kd + off, &ck_map, sl * 64, h, z, &kv_full[s]);
+                tma_load_3d(vd + off, &cv_map, sl * 64, h, z, &kv_full[s]);
+              }
+            }
+          }
+        }
+        ++it;
+      }
+      // every issued copy has landed before shared memory can go away
+      const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
+      bool late = false;
+      for (uint32_t j = first; j < it; ++j)
+        wait_or_abort(&kv_full[j % STAGES], (j / STAGES) & 1u, p.err, late);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- mma issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_qk = idesc_bf16_f32(128, BN, false);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, true);
+      const uint32_t tO = tmem + 2 * BN;
+      const uint32_t q_base = smem_u32(sQ);
+      const uint32_t p_base = smem_u32(sP);
+      wait_or_abort(q_full, 0, p.err, aborted);
+      auto issue_pv = [&](uint32_t jj) {
+        const int pb = jj & 1;
+        if (wait_or_abort(&p_full[pb], (jj >> 1) & 1u, p.err, aborted)) {
+          tc_fence_after();
+          const uint32_t v_base = smem_u32(sStage + (jj % STAGES) * C::kStageBytes + C::kTileBytes);
+          const uint32_t pbuf = p_base + pb * C::kPBytes;
+#pragma unroll
+          for (int kk = 0; kk < BN / 16; ++kk) {
+            const uint64_t a = smem_desc_sw128(pbuf + (kk >> 2) * C::kPSlab + (kk & 3) * 32, 16, 1024);
+            const uint64_t bd = smem_desc_sw128(v_base + kk * 2048, C::kKVSlab, 1024);
+            umma_bf16(tO, a, bd, idesc_pv, (jj > 0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit(&pv_done[pb]);
+          umma_commit(&kv_empty[jj % STAGES]);
+        }
+      };
+      uint32_t j = 0;
+      int hist;
+      int64_t j0;
+      while (seq.next(hist, j0)) {
+        const int s = j % STAGES;
+        const int sb = j & 1;
+        bool ok = wait_or_abort(&kv_full[s], (j / STAGES) & 1u, p.err, aborted);
+        ok = ok && wait_or_abort(&s_free[sb], ((j >> 1) & 1u) ^ 1u, p.err, aborted);
+        if (ok) {
+          tc_fence_after();
+          const uint32_t k_base = smem_u32(sStage + s * C::kStageBytes);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint64_t a = smem_desc_sw128(q_base + (kk >> 2) * C::kQSlab + (kk & 3) * 32, 16, 1024);
+            const uint64_t bd = smem_desc_sw128(k_base + (kk >> 2) * C::kKVSlab + (kk & 3) * 32, 16, 1024);
+            umma_bf16(tmem + sb * BN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
+          }
+          umma_commit(&s_full[sb]);
+        }
+        if (j >= 1) issue_pv(j - 1);
+        ++j;
+      }
+      if (j >= 1) issue_pv(j - 1);
+      if (!aborted) umma_commit(o_full);
+      // every mma issued has finished before TMEM is released
+      umma_commit(drain);
+      bool late = false;
+      wait_or_abort(drain, 0, p.err, late);
+    }
+  } else {
+    // ---------------------------------------------------------------- softmax
+    const int quarter = warp & 3;  // TMEM lanes this warp may access
+    const int r = quarter * 32 + lane;
+    const int64_t pr = p0 + r / G;
+    const bool row_ok = r < rows_valid && pr <= p_last;
+    const int qh = h * G + r % G;
+    const int64_t W = u.window;
+    const int64_t lo_r = W == 0 ? 0 : (pr - W + 1 > 0 ? pr - W + 1 : 0);  // first visible key
+    const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
+    const float c = p.scale_log2;
+    float m_used = -INFINITY, l = 0.f;  // running max (log2 units) and sum of weights
+    uint32_t j = 0;
+    int hist;
+    int64_t j0;
+    auto clampi = [](int64_t v) -> int { return (int)(v < -1 ? -1 : (v > BN + 1 ? BN + 1 : v)); };
+    while (seq.next(hist, j0)) {
+      const int sb = j & 1;
+      // columns e of this tile visible to row pr: [a0, b0) U [a1, b1)
+      int a0 = 0, b0 = 0, a1 = 0, b1 = 0;
+      if (row_ok) {
+        if (!hist) {  // chunk keys at positions t0 + j0 + e, held while j0 + e < n
+          const int64_t hi = min(pr - t0 - j0, p.n - 1 - j0);  // causal, held
+          a0 = clampi(lo_r - t0 - j0);
+          b0 = clampi(hi + 1);
+        } else if (t0 <= u.cap) {  // ring not yet wrapped: slot j holds position j
+          a0 = clampi(lo_r - j0);
+          b0 = clampi(seq.n_hist - j0);
+        } else {  // wrapped: slots < r0 hold the newest run, slots >= r0 the older one
+          const int64_t A = lo_r - t0 + seq.r0;  // first visible slot of the newest run
+          a0 = clampi(A - j0);
+          b0 = clampi(seq.r0 - j0);
+          a1 = clampi(A + u.cap - j0);
+          b1 = clampi(u.cap - j0);
+        }
+      }
+      const bool full_vis = (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);
+      const bool warp_full = __all_sync(0xffffffffu, full_vis);  // warp-uniform fast path
+      if (warp_wait_or_abort(&s_full[sb], (j >> 1) & 1u, p.err, aborted)) tc_fence_after();
+      const uint32_t tS = t_lane + sb * BN;
+      // pass 1: row max of the visible logits (raw; scale > 0 so max(z) c = max(z c))
+      float mx;
+      {
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+        for (int cc = 0; cc < BN / 32; ++cc) {
+          uint32_t rr[32];
+          tmem_ld32(tS + cc * 32, rr);
+          tmem_ld_wait();
+          if (warp_full) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) m4[e & 3] = fmaxf(m4[e & 3], __uint_as_float(rr[e]));
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const int col = cc * 32 + e;
+              const bool vis = full_vis || (col >= a0 && col < b0) || (col >= a1 && col < b1);
+              m4[e & 3] = fmaxf(m4[e & 3], vis ? __uint_as_float(rr[e]) : -INFINITY);
+            }
+          }
+        }
+        mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * c;
+      }
+      const float m_new = fmaxf(m_used, mx);
+      const bool resc = m_new - m_used > 8.f;  // false while both are -inf
+      float alpha = 1.f;
+      if (resc) {
+        alpha = ex2(m_used - m_new);
+        m_used = m_new;
+        l *= alpha;
+      }
+      const float bias = m_used == -INFINITY ? 0.f : m_used;
+
+      // O holds PV of tiles < j once PV(j-1) is done: rescale it then (rare: the
+      // reference max only moves when a row's max grows by more than 2^8)
+      if (j >= 1 && __any_sync(0xffffffffu, resc)) {
+        if (warp_wait_or_abort(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1u, p.err, aborted))
+          tc_fence_after();
+        const uint32_t tO = t_lane + 2 * BN;
+#pragma unroll
+        for (int cc = 0; cc < D / 32; ++cc) {
+          uint32_t rr[32];
+          tmem_ld32(tO + cc * 32, rr);
+          tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
+          tmem_st32(tO + cc * 32, rr);
+        }
+        tmem_st_wait();
+      }
+      // P buffer j & 1 was last read by PV(j-2)
+      const int pb = j & 1;
+      if (j >= 2) warp_wait_or_abort(&pv_done[pb], ((j - 2) >> 1) & 1u, p.err, aborted);
+      uint8_t* pbuf = sP + pb * C::kPBytes;
+      // pass 2: weights 2^(z - m) -> bf16 P row in shared memory (128-byte swizzle,
+      // the K-major A operand of the PV mma); sum in fp32
+      float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int cc = 0; cc < BN / 32; ++cc) {
+        uint32_t rr[32];
+        tmem_ld32(tS + cc * 32, rr);
+        tmem_ld_wait();
+        float w[32];
+        if (warp_full) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            w[e] = ex2(fmaf(__uint_as_float(rr[e]), c, -bias));
+            s4[e & 3] += w[e];
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const int col = cc * 32 + e;
+            const bool vis = full_vis || (col >= a0 && col < b0) || (col >= a1 && col < b1);
+            w[e] = vis ? ex2(fmaf(__uint_as_float(rr[e]), c, -bias)) : 0.f;
+            s4[e & 3] += w[e];
+          }
+        }
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          const int ch = cc * 4 + q4;  // 16-byte chunk = 8 keys
+          uint4 v;
+          v.x = pack_bf16(w[q4 * 8 + 0], w[q4 * 8 + 1]);
+          v.y = pack_bf16(w[q4 * 8 + 2], w[q4 * 8 + 3]);
+          v.z = pack_bf16(w[q4 * 8 + 4], w[q4 * 8 + 5]);
+          v.w = pack_bf16(w[q4 * 8 + 6], w[q4 * 8 + 7]);
+          *reinterpret_cast<uint4*>(pbuf + (ch >> 3) * C::kPSlab + swz128(r, ch & 7)) = v;
+        }
+      }
+      const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+      l += sum;
+      tc_fence_before();
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&s_free[sb]);  // S tile fully read
+        mbar_arrive(&p_full[pb]);  // P row block written
+      }
+      ++j;
+    }
+    // epilogue: O / l for this row
+    if (warp_wait_or_abort(o_full, 0, p.err, aborted)) tc_fence_after();
+    const float inv = l > 0.f ? 1.f / l : 0.f;
+    float* dst = p.out + (((int64_t)b * p.n + (pr - t0)) * p.n_q_heads + qh) * D;
+#pragma unroll
+    for (int cc = 0; cc < D / 32; ++cc) {
+      uint32_t rr[32];
+      tmem_ld32(t_lane + 2 * BN + cc * 32, rr);
+      tmem_ld_wait();
+      if (row_ok) {
+#pragma unroll
+        for (int e = 0; e < 32; e += 4)
+          *reinterpret_cast<float4*>(dst + cc * 32 + e) =
+              make_float4(__uint_as_float(rr[e]) * inv, __uint_as_float(rr[e + 1]) * inv,
+                          __uint_as_float(rr[e + 2]) * inv, __uint_as_float(rr[e + 3]) * inv);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
+}
+
+template <int D, int BN, int STAGES>
+static cudaError_t launch_tc(const PrefillParams& p, const CUtensorMap& qm, const CUtensorMap& km,
+                             const CUtensorMap& vm, const CUtensorMap& rm, cudaStream_t s) {
+  using C = TcCfg<D, BN, STAGES>;
+  cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D, BN, STAGES>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+  if (e != cudaSuccess) return e;
+  const int QP = 128 / p.group;
+  dim3 grid((unsigned)((p.n + QP - 1) / QP), (unsigned)p.n_units, (unsigned)p.batch);
+  prefill_tc_kernel<D, BN, STAGES><<<grid, 192, C::kSmem, s>>>(qm, km, vm, rm, p);
+  return cudaGetLastError();
+}
+
+int prefill_tc_rows_per_tile(int group) { return (128 / group) * group; }
+
+cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtensorMap& q_map,
+                              const CUtensorMap& ck_map, const CUtensorMap& cv_map,
+                              const CUtensorMap& ring_map, cudaStream_t s) {
+  if (p.n == 0) return cudaSuccess;
+  switch (head_dim) {
+    case 64: return launch_tc<64, 128, 3>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 128: return launch_tc<128, 64, 4>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 256: return launch_tc<256, 64, 2>(p, q_map, ck_map, cv_map, ring_map, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace hwkv

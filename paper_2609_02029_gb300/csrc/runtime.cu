@@ -285,7 +285,8 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
   if (c->t[layer] + n > c->pol.max_ctx)
     return fail(HWKV_ECAPACITY, "layer %d: t=%lld + n=%lld exceeds max_ctx=%lld", layer,
                 (long long)c->t[layer], (long long)n, (long long)c->pol.max_ctx);
-  if (n > (int64_t)65535 * 64) return fail(HWKV_EUNSUPPORTED, "chunk of %lld tokens too long", (long long)n);
+  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
+  if (n > (int64_t)65535 * 16) return fail(HWKV_EUNSUPPORTED, "chunk of %lld tokens too long", (long long)n);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   PrefillParams p{};
   p.n_units = c->pol.n_kv_heads;
@@ -306,7 +307,38 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
     p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window};
   }
-  cudaError_t e = launch_prefill(p, c->pol.head_dim, s);
+  // tensor maps of this call's q and chunk K/V: 3-D views {d, heads, batch * n}
+  auto encode = get_encode();
+  const int d = c->pol.head_dim, G = p.group, QP = 128 / G;
+  const cuuint32_t estr[3] = {1, 1, 1};
+  CUtensorMap q_map, ck_map, cv_map;
+  {
+    const cuuint64_t dim[3] = {(cuuint64_t)d, (cuuint64_t)c->pol.n_q_heads,
+                               (cuuint64_t)c->pol.batch * (cuuint64_t)n};
+    const cuuint64_t str[2] = {(cuuint64_t)d * 2, (cuuint64_t)c->pol.n_q_heads * d * 2};
+    const cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)QP};
+    CUresult r = encode(&q_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dim, str,
+                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(HWKV_EINVAL, "q tensor map rejected (%d): q must be 16-byte aligned", (int)r);
+  }
+  {
+    const cuuint64_t dim[3] = {(cuuint64_t)d, (cuuint64_t)c->pol.n_kv_heads,
+                               (cuuint64_t)c->pol.batch * (cuuint64_t)n};
+    const cuuint64_t str[2] = {(cuuint64_t)d * 2, (cuuint64_t)c->pol.n_kv_heads * d * 2};
+    const cuuint32_t box[3] = {64, 1, 64};
+    CUresult r = encode(&ck_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(k), dim,
+                        str, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r == CUDA_SUCCESS)
+      r = encode(&cv_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(v), dim, str,
+                 box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(HWKV_EINVAL, "k/v tensor map rejected (%d): k/v must be 16-byte aligned", (int)r);
+  }
+  if ((int64_t)c->pol.batch * n + 128 >= (int64_t)INT32_MAX)
+    return fail(HWKV_EUNSUPPORTED, "batch x chunk exceeds the TMA coordinate range");
+  cudaError_t e = launch_prefill_tc(p, d, q_map, ck_map, cv_map, c->kv_map, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "prefill launch: %s", cudaGetErrorString(e));
   // attend first, then write the chunk's retained tokens (stream order)
   const AppendParams ap = append_params(c, layer, k, v, n);
@@ -379,6 +411,7 @@ hwkv_status hwkv_decode_attn(hwkv_cache* c, int32_t layer, const void* q, float 
   hwkv_status st = check_layer(c, layer);
   if (st != HWKV_OK) return st;
   if (!q || !out) return fail(HWKV_EINVAL, "q/out is NULL");
+  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
   if (c->t[layer] <= 0) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
   if (c->t[layer] > INT32_MAX) return fail(HWKV_EUNSUPPORTED, "ring longer than 2^31");
   DecodeParams p{};

@@ -89,6 +89,10 @@ def test_decode_multi_layer_independent_state():
     (128, 8, 4, 2, [0, 1, 50, 100], [100, 37, 200, 64]),   # chunk > window, ragged
     (256, 12, 2, 1, [0, 130], [70, 130, 129, 1]),          # wrap inside history
     (128, 4, 1, 2, [64], [64, 64, 65, 63]),
+    (64, 3, 3, 1, [0, 200, 7], [300, 129]),                # G=1: 128 positions per tile
+    (128, 16, 2, 1, [0, 90], [257, 100]),                  # G=8
+    (64, 9, 3, 2, [0, 150, 33], [190, 70]),                # G=3: 126 valid rows of 128
+    (256, 10, 2, 1, [0, 77], [140, 60]),                   # G=5: 125 valid rows
 ])
 def test_prefill_parity(d, Hq, Hkv, B, windows, chunks):
     total = sum(chunks)
