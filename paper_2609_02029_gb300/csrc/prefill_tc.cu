@@ -16,8 +16,10 @@
 //   warp 0      TMA producer: Q once, then K/V tiles into a STAGES-deep ring
 //   warp 1      MMA issuer (one thread): S = Q K^T into a double-buffered TMEM
 //               tile (128 x BN fp32), then O += P V into TMEM (128 x D fp32)
-//   warps 2-5   softmax: thread r owns TMEM lane r = query row r, so the row
-//               max and sum are thread-local; P goes to shared memory as bf16
+//   warps 2+    softmax: thread r owns TMEM lane r = query row r, so the row
+//               max and sum are thread-local (at head_dim <= 128 two warps
+//               share each row quarter, splitting its columns and exchanging
+//               the row max through shared memory); P goes to shared memory as bf16
 //               (128-byte swizzle) for the PV mma; O is rescaled in TMEM only
 //               when a row's running max grows by more than 2^8 (the final
 //               O / l uses the same reference, so the result is exact).
@@ -30,8 +32,13 @@ namespace hwkv {
 
 namespace {
 
-template <int D, int BN, int STAGES>
+template <int D, int BN, int STAGES, int SPLIT>
 struct TcCfg {
+  static constexpr int kSoftmaxWarps = 4 * SPLIT;  // SPLIT warps share each TMEM lane quarter
+  static constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
+  static constexpr int kCW = BN / SPLIT;           // S columns per softmax warp
+  static constexpr int kOW = D / SPLIT;            // O columns per softmax warp
+  static_assert(kCW % 32 == 0 && kOW % 32 == 0, "column split");
   static constexpr int kSlabs = D / 64;
   static constexpr int kQSlab = 128 * 128;             // 128 rows x 128 B
   static constexpr int kQBytes = kSlabs * kQSlab;
@@ -39,9 +46,11 @@ struct TcCfg {
   static constexpr int kTileBytes = kSlabs * kKVSlab;  // one K (or V) tile
   static constexpr int kStageBytes = 2 * kTileBytes;
   static constexpr int kPSlab = 128 * 128;             // P: 128 rows x 64 keys
-  static constexpr int kPBytes = (BN / 64) * kPSlab;  // one P buffer; two are kept
+  static constexpr int kPBytes = (BN / 64) * kPSlab;  // the P buffer
   static constexpr int kBarBytes = 256;
-  static constexpr int kSmem = kQBytes + STAGES * kStageBytes + 2 * kPBytes + kBarBytes + 1024;
+  static constexpr int kRedBytes = SPLIT > 1 ? 2 * 2 * 128 * 4 : 0;  // row-max exchange
+  static constexpr int kSmem =
+      kQBytes + STAGES * kStageBytes + kPBytes + kBarBytes + kRedBytes + 1024;
   static constexpr uint32_t kTmemCols = 512;
   static_assert(2 * BN + D <= 512, "TMEM: two S buffers and O");
 };
@@ -126,7 +135,7 @@ struct KeySeq {
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, int* err,
                                               bool& aborted) {
   if (aborted) return false;
-  if (!mbar_wait_sleep_bounded(bar, parity, err)) aborted = true;
+  if (!mbar_wait_bounded(bar, parity, err)) aborted = true;
   return !aborted;
 }
 
@@ -143,30 +152,31 @@ __device__ __forceinline__ bool warp_wait_or_abort(uint64_t* bar, uint32_t parit
 
 }  // namespace
 
-template <int D, int BN, int STAGES>
-__global__ void __launch_bounds__(192, 1)
+template <int D, int BN, int STAGES, int SPLIT>
+__global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
     prefill_tc_kernel(const __grid_constant__ CUtensorMap q_map,
                       const __grid_constant__ CUtensorMap ck_map,
                       const __grid_constant__ CUtensorMap cv_map,
                       const __grid_constant__ CUtensorMap ring_map, const PrefillParams p) {
-  using C = TcCfg<D, BN, STAGES>;
+  using C = TcCfg<D, BN, STAGES, SPLIT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* sQ = smem;
   uint8_t* sStage = smem + C::kQBytes;
-  uint8_t* sP = sStage + STAGES * C::kStageBytes;  // [2] P buffers
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * C::kPBytes);
+  uint8_t* sP = sStage + STAGES * C::kStageBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + C::kPBytes);
   uint64_t* kv_full = bars;              // [STAGES] TMA landed
   uint64_t* kv_empty = bars + STAGES;    // [STAGES] PV of that tile done
   uint64_t* s_full = bars + 2 * STAGES;  // [2] S tile computed
   uint64_t* s_free = s_full + 2;         // [2] S tile read by the softmax warps
-  uint64_t* p_full = s_free + 2;         // [2] P buffer written (and O rescaled)
-  uint64_t* pv_done = p_full + 2;        // [2] PV mma that read that P buffer done
-  uint64_t* q_full = pv_done + 2;
+  uint64_t* p_full = s_free + 2;         // P of the current tile written (and O rescaled)
+  uint64_t* pv_done = p_full + 1;        // PV mma of the previous tile done
+  uint64_t* q_full = pv_done + 1;
   uint64_t* o_full = q_full + 1;
   uint64_t* drain = o_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + C::kBarBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = p.group;
@@ -188,10 +198,10 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 4);  // one arrival per softmax warp
-      mbar_init(&p_full[i], 4);
-      mbar_init(&pv_done[i], 1);
+      mbar_init(&s_free[i], C::kSoftmaxWarps);  // one arrival per softmax warp
     }
+    mbar_init(p_full, C::kSoftmaxWarps);
+    mbar_init(pv_done, 1);
     mbar_init(q_full, 1);
     mbar_init(o_full, 1);
     mbar_init(drain, 1);
@@ -268,18 +278,17 @@ __global__ void __launch_bounds__(192, 1)
       const uint32_t p_base = smem_u32(sP);
       wait_or_abort(q_full, 0, p.err, aborted);
       auto issue_pv = [&](uint32_t jj) {
-        const int pb = jj & 1;
-        if (wait_or_abort(&p_full[pb], (jj >> 1) & 1u, p.err, aborted)) {
+        if (wait_or_abort(p_full, jj & 1u, p.err, aborted)) {
           tc_fence_after();
           const uint32_t v_base = smem_u32(sStage + (jj % STAGES) * C::kStageBytes + C::kTileBytes);
-          const uint32_t pbuf = p_base + pb * C::kPBytes;
+          const uint32_t pbuf = p_base;
 #pragma unroll
           for (int kk = 0; kk < BN / 16; ++kk) {
             const uint64_t a = smem_desc_sw128(pbuf + (kk >> 2) * C::kPSlab + (kk & 3) * 32, 16, 1024);
             const uint64_t bd = smem_desc_sw128(v_base + kk * 2048, C::kKVSlab, 1024);
             umma_bf16(tO, a, bd, idesc_pv, (jj > 0 || kk > 0) ? 1u : 0u);
           }
-          umma_commit(&pv_done[pb]);
+          umma_commit(pv_done);
           umma_commit(&kv_empty[jj % STAGES]);
         }
       };
@@ -314,8 +323,11 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else {
     // ---------------------------------------------------------------- softmax
-    const int quarter = warp & 3;  // TMEM lanes this warp may access
+    const int quarter = warp & 3;        // TMEM lanes this warp may access
+    const int half = (warp - 2) >> 2;     // which share of the columns (SPLIT = 2)
     const int r = quarter * 32 + lane;
+    const int cbase = half * C::kCW;      // first S column of this warp
+    const int obase = half * C::kOW;      // first O column of this warp
     const int64_t pr = p0 + r / G;
     const bool row_ok = r < rows_valid && pr <= p_last;
     const int qh = h * G + r % G;
@@ -351,29 +363,40 @@ __global__ void __launch_bounds__(192, 1)
       const bool full_vis = (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);
       const bool warp_full = __all_sync(0xffffffffu, full_vis);  // warp-uniform fast path
       if (warp_wait_or_abort(&s_full[sb], (j >> 1) & 1u, p.err, aborted)) tc_fence_after();
-      const uint32_t tS = t_lane + sb * BN;
-      // pass 1: row max of the visible logits (raw; scale > 0 so max(z) c = max(z c))
+      // this warp's S columns, read once into registers; the S buffer is then free
+      // for the QK^T of tile j + 2 while this tile's softmax runs
+      uint32_t sv[C::kCW];
+#pragma unroll
+      for (int cc = 0; cc < C::kCW / 32; ++cc)
+        tmem_ld32(t_lane + sb * BN + cbase + cc * 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[cc * 32]));
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);
+      // row max of the visible logits (raw; scale > 0 so max(z) c = max(z c))
       float mx;
       {
         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        if (warp_full) {
 #pragma unroll
-        for (int cc = 0; cc < BN / 32; ++cc) {
-          uint32_t rr[32];
-          tmem_ld32(tS + cc * 32, rr);
-          tmem_ld_wait();
-          if (warp_full) {
+          for (int e = 0; e < C::kCW; ++e) m4[e & 3] = fmaxf(m4[e & 3], __uint_as_float(sv[e]));
+        } else {
 #pragma unroll
-            for (int e = 0; e < 32; ++e) m4[e & 3] = fmaxf(m4[e & 3], __uint_as_float(rr[e]));
-          } else {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const int col = cc * 32 + e;
-              const bool vis = full_vis || (col >= a0 && col < b0) || (col >= a1 && col < b1);
-              m4[e & 3] = fmaxf(m4[e & 3], vis ? __uint_as_float(rr[e]) : -INFINITY);
-            }
+          for (int e = 0; e < C::kCW; ++e) {
+            const int col = cbase + e;
+            const bool vis = full_vis || (col >= a0 && col < b0) || (col >= a1 && col < b1);
+            if (!vis) sv[e] = __float_as_uint(-INFINITY);
+            m4[e & 3] = fmaxf(m4[e & 3], __uint_as_float(sv[e]));
           }
         }
-        mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * c;
+        mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        if (SPLIT > 1) {  // combine with the warp holding the other columns of these rows
+          float* rb = red + (j & 1) * 256;
+          rb[half * 128 + r] = mx;
+          asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");
+          mx = fmaxf(mx, rb[(1 - half) * 128 + r]);
+        }
+        mx *= c;
       }
       const float m_new = fmaxf(m_used, mx);
       const bool resc = m_new - m_used > 8.f;  // false while both are -inf
@@ -385,14 +408,24 @@ __global__ void __launch_bounds__(192, 1)
       }
       const float bias = m_used == -INFINITY ? 0.f : m_used;
 
-      // O holds PV of tiles < j once PV(j-1) is done: rescale it then (rare: the
-      // reference max only moves when a row's max grows by more than 2^8)
-      if (j >= 1 && __any_sync(0xffffffffu, resc)) {
-        if (warp_wait_or_abort(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1u, p.err, aborted))
-          tc_fence_after();
-        const uint32_t tO = t_lane + 2 * BN;
+      // weights 2^(z c - m), computed in place (masked logits are -inf: weight 0)
+      float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int cc = 0; cc < D / 32; ++cc) {
+      for (int e = 0; e < C::kCW; ++e) {
+        const float w = ex2(fmaf(__uint_as_float(sv[e]), c, -bias));
+        s4[e & 3] += w;
+        sv[e] = __float_as_uint(w);
+      }
+      const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+
+      // PV of the previous tile has read P and added into O: only now may P be
+      // overwritten and O rescaled (rare: the reference max only moves when a
+      // row's max grows by more than 2^8)
+      if (j >= 1 && warp_wait_or_abort(pv_done, (j - 1) & 1u, p.err, aborted)) tc_fence_after();
+      if (j >= 1 && __any_sync(0xffffffffu, resc)) {
+        const uint32_t tO = t_lane + 2 * BN + obase;
+#pragma unroll
+        for (int cc = 0; cc < C::kOW / 32; ++cc) {
           uint32_t rr[32];
           tmem_ld32(tO + cc * 32, rr);
           tmem_ld_wait();
@@ -402,64 +435,37 @@ __global__ void __launch_bounds__(192, 1)
         }
         tmem_st_wait();
       }
-      // P buffer j & 1 was last read by PV(j-2)
-      const int pb = j & 1;
-      if (j >= 2) warp_wait_or_abort(&pv_done[pb], ((j - 2) >> 1) & 1u, p.err, aborted);
-      uint8_t* pbuf = sP + pb * C::kPBytes;
-      // pass 2: weights 2^(z - m) -> bf16 P row in shared memory (128-byte swizzle,
-      // the K-major A operand of the PV mma); sum in fp32
-      float s4[4] = {0.f, 0.f, 0.f, 0.f};
+      // P row -> shared memory, bf16, 128-byte swizzle (the K-major A operand of PV)
 #pragma unroll
-      for (int cc = 0; cc < BN / 32; ++cc) {
-        uint32_t rr[32];
-        tmem_ld32(tS + cc * 32, rr);
-        tmem_ld_wait();
-        float w[32];
-        if (warp_full) {
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            w[e] = ex2(fmaf(__uint_as_float(rr[e]), c, -bias));
-            s4[e & 3] += w[e];
-          }
-        } else {
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int col = cc * 32 + e;
-            const bool vis = full_vis || (col >= a0 && col < b0) || (col >= a1 && col < b1);
-            w[e] = vis ? ex2(fmaf(__uint_as_float(rr[e]), c, -bias)) : 0.f;
-            s4[e & 3] += w[e];
-          }
-        }
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          const int ch = cc * 4 + q4;  // 16-byte chunk = 8 keys
-          uint4 v;
-          v.x = pack_bf16(w[q4 * 8 + 0], w[q4 * 8 + 1]);
-          v.y = pack_bf16(w[q4 * 8 + 2], w[q4 * 8 + 3]);
-          v.z = pack_bf16(w[q4 * 8 + 4], w[q4 * 8 + 5]);
-          v.w = pack_bf16(w[q4 * 8 + 6], w[q4 * 8 + 7]);
-          *reinterpret_cast<uint4*>(pbuf + (ch >> 3) * C::kPSlab + swz128(r, ch & 7)) = v;
-        }
+      for (int ch8 = 0; ch8 < C::kCW / 8; ++ch8) {
+        const int ch = (cbase >> 3) + ch8;  // 16-byte chunk = 8 keys
+        uint4 v;
+        v.x = pack_bf16(__uint_as_float(sv[ch8 * 8 + 0]), __uint_as_float(sv[ch8 * 8 + 1]));
+        v.y = pack_bf16(__uint_as_float(sv[ch8 * 8 + 2]), __uint_as_float(sv[ch8 * 8 + 3]));
+        v.z = pack_bf16(__uint_as_float(sv[ch8 * 8 + 4]), __uint_as_float(sv[ch8 * 8 + 5]));
+        v.w = pack_bf16(__uint_as_float(sv[ch8 * 8 + 6]), __uint_as_float(sv[ch8 * 8 + 7]));
+        *reinterpret_cast<uint4*>(sP + (ch >> 3) * C::kPSlab + swz128(r, ch & 7)) = v;
       }
-      const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
       l += sum;
       tc_fence_before();
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&s_free[sb]);  // S tile fully read
-        mbar_arrive(&p_full[pb]);  // P row block written
-      }
+      if (lane == 0) mbar_arrive(p_full);  // P rows written (and O rescaled)
       ++j;
     }
     // epilogue: O / l for this row
     if (warp_wait_or_abort(o_full, 0, p.err, aborted)) tc_fence_after();
+    if (SPLIT > 1) {  // each warp of the pair summed only its columns
+      red[half * 128 + r] = l;  // every max exchange was read before o_full
+      asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");
+      l += red[(1 - half) * 128 + r];
+    }
     const float inv = l > 0.f ? 1.f / l : 0.f;
-    float* dst = p.out + (((int64_t)b * p.n + (pr - t0)) * p.n_q_heads + qh) * D;
+    float* dst = p.out + (((int64_t)b * p.n + (pr - t0)) * p.n_q_heads + qh) * D + obase;
 #pragma unroll
-    for (int cc = 0; cc < D / 32; ++cc) {
+    for (int cc = 0; cc < C::kOW / 32; ++cc) {
       uint32_t rr[32];
-      tmem_ld32(t_lane + 2 * BN + cc * 32, rr);
+      tmem_ld32(t_lane + 2 * BN + obase + cc * 32, rr);
       tmem_ld_wait();
       if (row_ok) {
 #pragma unroll
@@ -477,16 +483,16 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
 }
 
-template <int D, int BN, int STAGES>
+template <int D, int BN, int STAGES, int SPLIT>
 static cudaError_t launch_tc(const PrefillParams& p, const CUtensorMap& qm, const CUtensorMap& km,
                              const CUtensorMap& vm, const CUtensorMap& rm, cudaStream_t s) {
-  using C = TcCfg<D, BN, STAGES>;
-  cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D, BN, STAGES>,
+  using C = TcCfg<D, BN, STAGES, SPLIT>;
+  cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D, BN, STAGES, SPLIT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
   if (e != cudaSuccess) return e;
   const int QP = 128 / p.group;
   dim3 grid((unsigned)((p.n + QP - 1) / QP), (unsigned)p.n_units, (unsigned)p.batch);
-  prefill_tc_kernel<D, BN, STAGES><<<grid, 192, C::kSmem, s>>>(qm, km, vm, rm, p);
+  prefill_tc_kernel<D, BN, STAGES, SPLIT><<<grid, C::kThreads, C::kSmem, s>>>(qm, km, vm, rm, p);
   return cudaGetLastError();
 }
 
@@ -497,9 +503,9 @@ cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtens
                               const CUtensorMap& ring_map, cudaStream_t s) {
   if (p.n == 0) return cudaSuccess;
   switch (head_dim) {
-    case 64: return launch_tc<64, 128, 3>(p, q_map, ck_map, cv_map, ring_map, s);
-    case 128: return launch_tc<128, 64, 4>(p, q_map, ck_map, cv_map, ring_map, s);
-    case 256: return launch_tc<256, 64, 2>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 64: return launch_tc<64, 128, 3, 2>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 128: return launch_tc<128, 128, 2, 2>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 256: return launch_tc<256, 64, 2, 1>(p, q_map, ck_map, cv_map, ring_map, s);
     default: return cudaErrorInvalidValue;
   }
 }
