@@ -19,8 +19,8 @@
 //   warps 2+    softmax: thread r owns TMEM lane r = query row r, so the row
 //               max and sum are thread-local (at head_dim <= 128 two warps
 //               share each row quarter, splitting its columns and exchanging
-//               the row max through shared memory); P goes to shared memory as bf16
-//               (128-byte swizzle) for the PV mma; O is rescaled in TMEM only
+//               the row max through shared memory); P goes back to TMEM as bf16
+//               and is the tensor-memory A operand of the PV mma; O is rescaled in TMEM only
 //               when a row's running max grows by more than 2^8 (the final
 //               O / l uses the same reference, so the result is exact).
 // While the softmax warps work on tile j the tensor core computes S of tile j+1.
@@ -45,14 +45,15 @@ struct TcCfg {
   static constexpr int kKVSlab = BN * 128;             // BN rows x 128 B
   static constexpr int kTileBytes = kSlabs * kKVSlab;  // one K (or V) tile
   static constexpr int kStageBytes = 2 * kTileBytes;
-  static constexpr int kPSlab = 128 * 128;             // P: 128 rows x 64 keys
-  static constexpr int kPBytes = (BN / 64) * kPSlab;  // the P buffer
+  // TMEM columns: S0 [0, BN), S1 [BN, 2BN), O [2BN, 2BN + D), P [2BN + D, 2BN + D + BN/2)
+  static constexpr int kColO = 2 * BN;
+  static constexpr int kColP = 2 * BN + D;
   static constexpr int kBarBytes = 256;
   static constexpr int kRedBytes = SPLIT > 1 ? 2 * 2 * 128 * 4 : 0;  // row-max exchange
   static constexpr int kSmem =
-      kQBytes + STAGES * kStageBytes + kPBytes + kBarBytes + kRedBytes + 1024;
+      kQBytes + STAGES * kStageBytes + kBarBytes + kRedBytes + 1024;
   static constexpr uint32_t kTmemCols = 512;
-  static_assert(2 * BN + D <= 512, "TMEM: two S buffers and O");
+  static_assert(2 * BN + D + BN / 2 <= 512, "TMEM: two S buffers, O and P");
 };
 
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int32_t x,
@@ -164,8 +165,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
                                              ~uintptr_t(1023));
   uint8_t* sQ = smem;
   uint8_t* sStage = smem + C::kQBytes;
-  uint8_t* sP = sStage + STAGES * C::kStageBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + C::kPBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + STAGES * C::kStageBytes);
   uint64_t* kv_full = bars;              // [STAGES] TMA landed
   uint64_t* kv_empty = bars + STAGES;    // [STAGES] PV of that tile done
   uint64_t* s_full = bars + 2 * STAGES;  // [2] S tile computed
@@ -273,20 +273,18 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, BN, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, true);
-      const uint32_t tO = tmem + 2 * BN;
+      const uint32_t tO = tmem + C::kColO;
+      const uint32_t tP = tmem + C::kColP;
       const uint32_t q_base = smem_u32(sQ);
-      const uint32_t p_base = smem_u32(sP);
       wait_or_abort(q_full, 0, p.err, aborted);
       auto issue_pv = [&](uint32_t jj) {
         if (wait_or_abort(p_full, jj & 1u, p.err, aborted)) {
           tc_fence_after();
           const uint32_t v_base = smem_u32(sStage + (jj % STAGES) * C::kStageBytes + C::kTileBytes);
-          const uint32_t pbuf = p_base;
 #pragma unroll
-          for (int kk = 0; kk < BN / 16; ++kk) {
-            const uint64_t a = smem_desc_sw128(pbuf + (kk >> 2) * C::kPSlab + (kk & 3) * 32, 16, 1024);
+          for (int kk = 0; kk < BN / 16; ++kk) {  // 16 keys = 8 packed P columns
             const uint64_t bd = smem_desc_sw128(v_base + kk * 2048, C::kKVSlab, 1024);
-            umma_bf16(tO, a, bd, idesc_pv, (jj > 0 || kk > 0) ? 1u : 0u);
+            umma_bf16_tmem_a(tO, tP + kk * 8, bd, idesc_pv, (jj > 0 || kk > 0) ? 1u : 0u);
           }
           umma_commit(pv_done);
           umma_commit(&kv_empty[jj % STAGES]);
@@ -423,7 +421,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
       // row's max grows by more than 2^8)
       if (j >= 1 && warp_wait_or_abort(pv_done, (j - 1) & 1u, p.err, aborted)) tc_fence_after();
       if (j >= 1 && __any_sync(0xffffffffu, resc)) {
-        const uint32_t tO = t_lane + 2 * BN + obase;
+        const uint32_t tO = t_lane + C::kColO + obase;
 #pragma unroll
         for (int cc = 0; cc < C::kOW / 32; ++cc) {
           uint32_t rr[32];
@@ -435,20 +433,24 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
         }
         tmem_st_wait();
       }
-      // P row -> shared memory, bf16, 128-byte swizzle (the K-major A operand of PV)
+      // P row -> TMEM as bf16 pairs (A operand of the PV mma, read from tensor memory)
+      {
+        uint32_t pk[C::kCW / 2];
 #pragma unroll
-      for (int ch8 = 0; ch8 < C::kCW / 8; ++ch8) {
-        const int ch = (cbase >> 3) + ch8;  // 16-byte chunk = 8 keys
-        uint4 v;
-        v.x = pack_bf16(__uint_as_float(sv[ch8 * 8 + 0]), __uint_as_float(sv[ch8 * 8 + 1]));
-        v.y = pack_bf16(__uint_as_float(sv[ch8 * 8 + 2]), __uint_as_float(sv[ch8 * 8 + 3]));
-        v.z = pack_bf16(__uint_as_float(sv[ch8 * 8 + 4]), __uint_as_float(sv[ch8 * 8 + 5]));
-        v.w = pack_bf16(__uint_as_float(sv[ch8 * 8 + 6]), __uint_as_float(sv[ch8 * 8 + 7]));
-        *reinterpret_cast<uint4*>(sP + (ch >> 3) * C::kPSlab + swz128(r, ch & 7)) = v;
+        for (int e = 0; e < C::kCW / 2; ++e)
+          pk[e] = pack_bf16(__uint_as_float(sv[2 * e]), __uint_as_float(sv[2 * e + 1]));
+        const uint32_t tPw = t_lane + C::kColP + (cbase >> 1);
+        if constexpr (C::kCW / 2 == 16) {
+          tmem_st16(tPw, *reinterpret_cast<const uint32_t(*)[16]>(pk));
+        } else {
+#pragma unroll
+          for (int cc = 0; cc < C::kCW / 64; ++cc)
+            tmem_st32(tPw + cc * 32, *reinterpret_cast<const uint32_t(*)[32]>(&pk[cc * 32]));
+        }
+        tmem_st_wait();
       }
       l += sum;
       tc_fence_before();
-      fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full);  // P rows written (and O rescaled)
       ++j;
@@ -465,7 +467,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
 #pragma unroll
     for (int cc = 0; cc < C::kOW / 32; ++cc) {
       uint32_t rr[32];
-      tmem_ld32(t_lane + 2 * BN + obase + cc * 32, rr);
+      tmem_ld32(t_lane + C::kColO + obase + cc * 32, rr);
       tmem_ld_wait();
       if (row_ok) {
 #pragma unroll
