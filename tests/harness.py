@@ -114,3 +114,25 @@ def assert_close(got, want, what=""):
     assert err.max() <= MAX_ABS, "%s: max abs err %.4g > %g" % (what, err.max(), MAX_ABS)
     assert err.mean() <= MEAN_ABS, "%s: mean abs err %.4g > %g" % (what, err.mean(), MEAN_ABS)
     return err.max(), err.mean()
+
+
+def oracle_unit_decode(run, layer, b, h, p):
+    """Oracle outputs [G, d] of the G query heads of KV head h at position p, from
+    host-generated inputs (array form: the K/V window is generated once)."""
+    W = run.window(layer, h)
+    Weff = 0 if (W == 0 or W >= run.max_ctx) else W
+    lo = oracle.window_lo(p, Weff)
+    K = hwkv_gen.fill_host_sub(run.g, hwkv_gen.K, layer, b, lo, p - lo + 1, h, 1, run.d)[:, 0]
+    V = hwkv_gen.fill_host_sub(run.g, hwkv_gen.V, layer, b, lo, p - lo + 1, h, 1, run.d)[:, 0]
+    Q = hwkv_gen.fill_host_sub(run.g, hwkv_gen.Q, layer, b, p, 1, h * run.G, run.G, run.d)[0]
+    O, sp = oracle.window_attention_bf16(Q, [p - lo] * run.G, K, V, 0, run.scale)
+    np.testing.assert_allclose(sp, 1.0, atol=1e-12)
+    return O
+
+
+def check_ring_unit(run, layer, b, h):
+    t = hwkv.hwkv_seq_len(run.cache, layer)
+    kr, vr = hwkv.hwkv_debug_copy_ring(run.cache, layer, b, h, run.d)
+    cap = kr.shape[0]
+    assert np.array_equal(kr, oracle.ring_expected_gen(run.g, hwkv_gen.K, layer, b, h, run.d, t, cap))
+    assert np.array_equal(vr, oracle.ring_expected_gen(run.g, hwkv_gen.V, layer, b, h, run.d, t, cap))
