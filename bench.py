@@ -33,6 +33,11 @@ sys.path.insert(0, ROOT)
 from hwkv_gen import workloads  # noqa: E402
 
 NOMINAL_HBM_GBS = 8000.0
+# DRAM bytes (read + write) per algorithmic byte of the decode split kernel, from the ncu
+# capture in profiles/decode_split_small_full.md (1 layer, batch 2 of layers16_112k);
+# traffic is reads of every resident K/V row plus tile partials, so it scales with the
+# algorithmic bytes of a launch. Set to None whenever that kernel changes.
+DECODE_TRAFFIC_PER_BYTE = (244.238336e6 + 3.453184e6) / 244066304.0
 
 
 def peaks():
@@ -592,7 +597,10 @@ def main():
                      "frac": r["achieved_gbs"] / hbm, "peak_source": peak_src,
                      "frac_of_nominal_8tbs": r["achieved_gbs"] / NOMINAL_HBM_GBS,
                      "bytes_per_launch": r["bytes_avg"], "launch_ms": r["dec_avg_ms"],
-                     "traffic": None},
+                     "traffic": (r["bytes_avg"] * DECODE_TRAFFIC_PER_BYTE
+                                 if DECODE_TRAFFIC_PER_BYTE else None),
+                     "traffic_source": "ncu dram bytes of a 1-layer batch-2 capture, scaled by "
+                                       "algorithmic bytes"},
         "append_ms_per_launch": r["app_avg_ms"],
         "residency_bytes": r["resid_bytes"],
         "e2e": {"value": r["e2e_value"], "unit": "tokens/s", "h2d_bytes_per_step": r["h2d"],
