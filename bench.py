@@ -33,8 +33,8 @@ sys.path.insert(0, ROOT)
 from hwkv_gen import workloads  # noqa: E402
 
 NOMINAL_HBM_GBS = 8000.0
-# DRAM bytes (read + write) per algorithmic byte of the decode split kernel, from the ncu
-# capture in profiles/decode_split_small_full.md (1 layer, batch 2 of layers16_112k);
+# DRAM bytes (read + write) per algorithmic byte of the decode split kernel, from an ncu
+# capture (--set full) of the 1-layer, batch-2 case of layers16_112k;
 # traffic is reads of every resident K/V row plus tile partials, so it scales with the
 # algorithmic bytes of a launch. Set to None whenever that kernel changes.
 DECODE_TRAFFIC_PER_BYTE = (244.238336e6 + 3.453184e6) / 244066304.0
