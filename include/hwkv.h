@@ -146,6 +146,21 @@ HWKV_API hwkv_status hwkv_prefill(hwkv_cache* cache, int32_t layer, const void* 
 HWKV_API hwkv_status hwkv_decode_attn(hwkv_cache* cache, int32_t layer, const void* q, float scale,
                              float* out, void* cuda_stream);
 
+/*
+ * One decode step of a layer in a single launch (+ the combine): appends the
+ * new token at position t (as hwkv_append with n = 1) and computes the decode
+ * attention of its queries (as hwkv_decode_attn after that append); then t += 1.
+ * The new token's K/V go straight from k_new/v_new into the attention and into
+ * ring slot t mod cap, which no other part of the step reads.
+ *   q:           [batch, n_q_heads, head_dim] bf16
+ *   k_new, v_new:[batch, n_kv_heads, head_dim] bf16
+ *   out:         [batch, n_q_heads, head_dim] fp32
+ * Fails with HWKV_ECAPACITY if t + 1 > max_ctx.
+ */
+HWKV_API hwkv_status hwkv_decode_step(hwkv_cache* cache, int32_t layer, const void* q,
+                                      const void* k_new, const void* v_new, float scale,
+                                      float* out, void* cuda_stream);
+
 /* Size of the device array hwkv_decode_attn_static keeps its scratch in. */
 #define HWKV_DECODE_STATIC_SCRATCH_BYTES (4u << 20)
 

@@ -68,6 +68,7 @@ def lib():
             "hwkv_prefill": [_vp, _i32, _vp, _vp, _vp, _i64, ctypes.c_float, _vp, _vp],
             "hwkv_decode_attn": [_vp, _i32, _vp, ctypes.c_float, _vp, _vp],
             "hwkv_decode_attn_static": [_vp, _i32, _vp, ctypes.c_float, _vp, _vp],
+            "hwkv_decode_step": [_vp, _i32, _vp, _vp, _vp, ctypes.c_float, _vp, _vp],
             "hwkv_residency_bytes": [_vp, _i32, _u64p],
             "hwkv_allocated_ring_bytes": [_vp, _i32, _u64p],
             "hwkv_seq_len": [_vp, _i32, ctypes.POINTER(_i64)],
@@ -152,6 +153,11 @@ def hwkv_prefill(cache, layer, q, k, v, n, scale, out, stream=None):
 
 def hwkv_decode_attn(cache, layer, q, scale, out, stream=None):
     _check(lib().hwkv_decode_attn(cache, layer, _ptr(q), scale, _ptr(out), _stream(stream)))
+
+
+def hwkv_decode_step(cache, layer, q, k_new, v_new, scale, out, stream=None):
+    _check(lib().hwkv_decode_step(cache, layer, _ptr(q), _ptr(k_new), _ptr(v_new), scale,
+                                  _ptr(out), _stream(stream)))
 
 
 def hwkv_decode_attn_static(cache, layer, q, scale, out, stream=None):

@@ -12,6 +12,8 @@
 namespace hwkv {
 
 __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
+  grid_dep_wait();  // k/v may come from the kernel launched before; the previous
+                    // decode of this ring must be done reading before slots are reused
   const int64_t vec_per_row = p.d / 8;
   const int64_t total = (int64_t)p.batch * p.n * p.n_units * vec_per_row;
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
@@ -42,8 +44,7 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
   int64_t blocks = (total + 255) / 256;
   const int64_t cap_blocks = 152 * 16;
   if (blocks > cap_blocks) blocks = cap_blocks;
-  append_kernel<<<(unsigned)blocks, 256, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(append_kernel, dim3((unsigned)blocks), dim3(256), 0, s, p);
 }
 
 }  // namespace hwkv

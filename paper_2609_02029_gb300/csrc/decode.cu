@@ -99,6 +99,8 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     fence_barrier_init();
   }
   __syncthreads();
+  grid_dep_wait();    // the ring append and q come from kernels launched before
+  grid_dep_launch();  // the combine kernel may start launching
 
   if (warp == kDecodeWarps) {
     // ------------------------------------------------------------ producer
@@ -182,6 +184,30 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
       }
       const uint32_t kbase = smem_u32(smem + s * C::kStageBytes);
       const uint32_t vbase = kbase + C::kTileBytes;
+      if (p.k_new != nullptr) {
+        // fused step: the new token's slot may lie in this stage; the warp owning that
+        // row replaces the staged (stale) row with the new K/V and writes the ring row
+        const int64_t row_in = (int64_t)p.u[ti.h].s_new - (ti.start + (int64_t)st * kStageTokens);
+        if (row_in >= w * 16 && row_in < w * 16 + 16) {
+          const int r = (int)row_in;
+          const __nv_bfloat16* src_k = p.k_new + ((int64_t)ti.b * p.n_units + ti.h) * D;
+          const __nv_bfloat16* src_v = p.v_new + ((int64_t)ti.b * p.n_units + ti.h) * D;
+          const int64_t ring_row = ti.k_row - ti.start + p.u[ti.h].s_new;  // K region row
+          const int64_t vring_row = ti.v_row - ti.start + p.u[ti.h].s_new;
+          for (int idx = lane; idx < 2 * (D / 8); idx += 32) {
+            const int isv = idx >= D / 8;
+            const int ch = isv ? idx - D / 8 : idx;  // 16-byte chunk of the row
+            const uint4 val = *reinterpret_cast<const uint4*>((isv ? src_v : src_k) + ch * 8);
+            const uint32_t dst = (isv ? vbase : kbase) + (ch >> 3) * kSlabBytes + swz128(r, ch & 7);
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(val.x),
+                         "r"(val.y), "r"(val.z), "r"(val.w)
+                         : "memory");
+            *reinterpret_cast<uint4*>(p.arena + (isv ? vring_row : ring_row) * D + ch * 8) = val;
+          }
+          fence_proxy_async_smem();  // this generic write precedes the next TMA into the stage
+          __syncwarp();
+        }
+      }
 
       // S^T = K . Q^T  (two accumulators to shorten the dependent mma chain)
       float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
@@ -307,20 +333,21 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
 }
 
 // Log-sum-exp merge of the tile partials of one (batch row, query head):
-// o = sum_j 2^{(m_j - M) c} o_j / sum_j 2^{(m_j - M) c} l_j, M = max_j m_j,
-// over the head's tiles in their fixed order (deterministic). One CTA per
-// (batch row, query head, 128-channel chunk); the tile weights are computed
-// once into shared memory, then each thread sums its channel over the tiles.
+// o = sum_j 2^{(m_j - M) c} o_j / sum_j 2^{(m_j - M) c} l_j, M = max_j m_j.
+// One CTA of 8 warps per (batch row, query head): warp w sums tiles w, w+8, ...
+// over all channels (each lane D/32 consecutive channels, vector loads); the
+// eight partial sums are added in shared memory in warp order (deterministic).
 // Heads whose ring is a single tile were written by the split kernel.
+constexpr int kCombineWarps = 8;
+
 template <int D>
-__global__ void __launch_bounds__(D < 128 ? D : 128) decode_combine_kernel(const DecodeParams p) {
-  constexpr int NT = D < 128 ? D : 128;
-  constexpr int CH = D / NT;
-  __shared__ float s_w[kCombineMaxTiles];
-  __shared__ float s_red[NT / 32];
-  __shared__ float s_bcast;
-  const int chunk = blockIdx.x % CH;
-  const int bq = blockIdx.x / CH;
+__global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(const DecodeParams p) {
+  constexpr int PER = D / 32;  // channels per lane
+  __shared__ float s_num[kCombineWarps][D];
+  __shared__ float s_den[kCombineWarps];
+  __shared__ float s_max[kCombineWarps];
+  grid_dep_wait();  // partials come from the split kernel launched before
+  const int bq = blockIdx.x;
   const int b = bq / p.n_q_heads;
   const int qh = bq - b * p.n_q_heads;
   const int h = qh / p.group;
@@ -330,55 +357,48 @@ __global__ void __launch_bounds__(D < 128 ? D : 128) decode_combine_kernel(const
   if (n_t <= 1) return;
   const int64_t tile0 = (int64_t)b * p.tiles_per_b + u.tile_begin;
   const float c = p.scale_log2;
-  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // M = max_j m_j
   float mx = -INFINITY;
-  for (int j = tid; j < n_t; j += NT) mx = fmaxf(mx, p.part_ml[(tile0 + j) * kMaxGroup + n].x);
+  for (int j = threadIdx.x; j < n_t; j += blockDim.x)
+    mx = fmaxf(mx, p.part_ml[(tile0 + j) * kMaxGroup + n].x);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  if (lane == 0) s_red[wid] = mx;
+  if (lane == 0) s_max[w] = mx;
   __syncthreads();
-  if (tid == 0) {
-    float m = s_red[0];
-    for (int k = 1; k < NT / 32; ++k) m = fmaxf(m, s_red[k]);
-    s_bcast = m;
-  }
-  __syncthreads();
-  const float M = s_bcast;
-  // weights and L = sum_j w_j l_j
-  float lsum = 0.f;
-  for (int j = tid; j < n_t; j += NT) {
+  float M = s_max[0];
+#pragma unroll
+  for (int k = 1; k < kCombineWarps; ++k) M = fmaxf(M, s_max[k]);
+
+  float acc[PER];
+#pragma unroll
+  for (int e = 0; e < PER; ++e) acc[e] = 0.f;
+  float den = 0.f;
+  for (int j = w; j < n_t; j += kCombineWarps) {
     const float2 ml = p.part_ml[(tile0 + j) * kMaxGroup + n];
-    const float wj = ml.x == -INFINITY ? 0.f : ex2((ml.x - M) * c);
-    s_w[j] = wj;
-    lsum += wj * ml.y;
+    const float wgt = ml.x == -INFINITY ? 0.f : ex2((ml.x - M) * c);
+    den += wgt * ml.y;
+    const float* src = p.part_o + ((tile0 + j) * kMaxGroup + n) * D + lane * PER;
+#pragma unroll
+    for (int e = 0; e < PER; e += 2) {
+      const float2 v = *reinterpret_cast<const float2*>(src + e);
+      acc[e] += wgt * v.x;
+      acc[e + 1] += wgt * v.y;
+    }
   }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+  for (int e = 0; e < PER; ++e) s_num[w][lane * PER + e] = acc[e];
+  if (lane == 0) s_den[w] = den;
   __syncthreads();
-  if (lane == 0) s_red[wid] = lsum;
-  __syncthreads();
-  if (tid == 0) {
-    float l = 0.f;
-    for (int k = 0; k < NT / 32; ++k) l += s_red[k];
-    s_bcast = l;
+  float dsum = 0.f;
+#pragma unroll
+  for (int k = 0; k < kCombineWarps; ++k) dsum += s_den[k];
+  for (int i = threadIdx.x; i < D; i += blockDim.x) {
+    float num = 0.f;
+#pragma unroll
+    for (int k = 0; k < kCombineWarps; ++k) num += s_num[k][i];
+    p.out[((int64_t)b * p.n_q_heads + qh) * D + i] = num / dsum;
   }
-  __syncthreads();
-  const float L = s_bcast;
-  const int i = chunk * NT + tid;
-  const float* src = p.part_o + (tile0 * kMaxGroup + n) * D + i;
-  const int64_t stride = (int64_t)kMaxGroup * D;
-  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-  int j = 0;
-  for (; j + 4 <= n_t; j += 4) {
-    a0 += s_w[j] * src[(j + 0) * stride];
-    a1 += s_w[j + 1] * src[(j + 1) * stride];
-    a2 += s_w[j + 2] * src[(j + 2) * stride];
-    a3 += s_w[j + 3] * src[(j + 3) * stride];
-  }
-  for (; j < n_t; ++j) a0 += s_w[j] * src[j * stride];
-  p.out[((int64_t)b * p.n_q_heads + qh) * D + i] = ((a0 + a1) + (a2 + a3)) / L;
 }
 
 int decode_smem_bytes(int head_dim) {
@@ -397,8 +417,8 @@ static cudaError_t launch_decode_t(const DecodeParams& p, const CUtensorMap& map
   cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  decode_split_kernel<D><<<grid, (kDecodeWarps + 1) * 32, smem, s>>>(map, p);
-  return cudaGetLastError();
+  return launch_pdl(decode_split_kernel<D>, dim3(grid), dim3((kDecodeWarps + 1) * 32), smem, s,
+                    map, p);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& map, int head_dim, int grid,
@@ -415,14 +435,13 @@ cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStrea
   bool any = false;  // nothing to merge when every ring is a single tile
   for (int h = 0; h < p.n_units; ++h) any |= p.u[h].n_tiles > 1;
   if (!any) return cudaSuccess;
-  const int bq = p.batch * p.n_q_heads;
+  const dim3 grid(p.batch * p.n_q_heads), block(kCombineWarps * 32);
   switch (head_dim) {
-    case 64: decode_combine_kernel<64><<<bq, 64, 0, s>>>(p); break;
-    case 128: decode_combine_kernel<128><<<bq, 128, 0, s>>>(p); break;
-    case 256: decode_combine_kernel<256><<<bq * 2, 128, 0, s>>>(p); break;
+    case 64: return launch_pdl(decode_combine_kernel<64>, grid, block, 0, s, p);
+    case 128: return launch_pdl(decode_combine_kernel<128>, grid, block, 0, s, p);
+    case 256: return launch_pdl(decode_combine_kernel<256>, grid, block, 0, s, p);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 }  // namespace hwkv

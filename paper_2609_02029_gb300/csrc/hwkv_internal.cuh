@@ -10,6 +10,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace hwkv {
 
 constexpr int kMaxKvHeads = 64;
@@ -31,7 +33,7 @@ struct DecodeUnit {
   int32_t n_valid;  // resident slots: min(t, cap)
   int32_t n_tiles;  // tiles this head's ring is split into, per batch row
   int32_t tile_begin;  // first tile of this head within one batch row's tile list
-  int32_t pad;
+  int32_t s_new;       // fused step: ring slot that receives the new token
 };
 
 struct DecodeParams {
@@ -48,6 +50,11 @@ struct DecodeParams {
   float2* part_ml;         // [n_tiles][kMaxGroup]: (max logit, sum of weights)
   float* out;              // [batch][n_q_heads][D]
   int* err;
+  // fused step (append the new token, then attend): k_new/v_new [batch][n_units][D];
+  // the new token's row is patched into the staged tile and written to the ring
+  const __nv_bfloat16* k_new;  // null: plain decode over the current ring contents
+  const __nv_bfloat16* v_new;
+  __nv_bfloat16* arena;        // K/V rows: row r at arena + r * D
   DecodeUnit u[kMaxKvHeads];
 };
 
@@ -101,6 +108,34 @@ int decode_smem_bytes(int head_dim);
 
 // ------------------------------------------------------------ device PTX
 #if defined(__CUDACC__)
+
+// Launch with programmatic dependent launch: the kernel may start while the
+// previous kernel of the stream finishes; it must call grid_dep_wait() before
+// touching memory that kernel wrote (and before overwriting memory it reads).
+template <typename... KArgs, typename... Args>
+static inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                     cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// wait until the grids this launch depends on have completed and their writes are visible
+__device__ __forceinline__ void grid_dep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+// allow the next programmatically dependent launch to begin launching
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

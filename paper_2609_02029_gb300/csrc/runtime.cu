@@ -352,9 +352,8 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
 // (batch row, KV head) ring. The length is chosen to balance the persistent
 // grid: minimise (tiles per CTA) x (tile length + a fixed per-tile cost).
 static void plan_decode(const hwkv_cache* c, int32_t layer, int max_tiles, DecodeParams& p,
-                        int& grid) {
+                        int& grid, int64_t t) {
   const int H = c->pol.n_kv_heads, B = c->pol.batch;
-  const int64_t t = c->t[layer];
   int64_t n_valid[kMaxKvHeads];
   int64_t longest = 0;
   for (int h = 0; h < H; ++h) {
@@ -397,7 +396,7 @@ static void plan_decode(const hwkv_cache* c, int32_t layer, int max_tiles, Decod
     du.n_valid = (int32_t)n_valid[h];
     du.n_tiles = (int32_t)((n_valid[h] + best_len - 1) / best_len);
     du.tile_begin = begin;
-    du.pad = 0;
+    du.s_new = (int32_t)((t - 1) % u.cap);  // slot of the newest token (fused step)
     begin += du.n_tiles;
   }
   p.tiles_per_b = begin;
@@ -426,7 +425,7 @@ hwkv_status hwkv_decode_attn(hwkv_cache* c, int32_t layer, const void* q, float 
   p.out = out;
   p.err = c->err();
   int grid = 0;
-  plan_decode(c, layer, c->lay.max_tiles, p, grid);
+  plan_decode(c, layer, c->lay.max_tiles, p, grid, c->t[layer]);
   if (p.n_tiles > c->lay.max_tiles)
     return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
@@ -434,6 +433,43 @@ hwkv_status hwkv_decode_attn(hwkv_cache* c, int32_t layer, const void* q, float 
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
   e = launch_decode_combine(p, c->pol.head_dim, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
+  return ok();
+}
+
+hwkv_status hwkv_decode_step(hwkv_cache* c, int32_t layer, const void* q, const void* k_new,
+                             const void* v_new, float scale, float* out, void* cuda_stream) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (!q || !out || !k_new || !v_new) return fail(HWKV_EINVAL, "q/k_new/v_new/out is NULL");
+  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
+  if (c->t[layer] + 1 > c->pol.max_ctx)
+    return fail(HWKV_ECAPACITY, "layer %d: t=%lld + 1 exceeds max_ctx=%lld", layer,
+                (long long)c->t[layer], (long long)c->pol.max_ctx);
+  if (c->t[layer] + 1 > INT32_MAX) return fail(HWKV_EUNSUPPORTED, "ring longer than 2^31");
+  DecodeParams p{};
+  p.n_units = c->pol.n_kv_heads;
+  p.batch = c->pol.batch;
+  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
+  p.n_q_heads = c->pol.n_q_heads;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.part_o = c->part_o();
+  p.part_ml = c->part_ml();
+  p.out = out;
+  p.err = c->err();
+  p.k_new = static_cast<const __nv_bfloat16*>(k_new);
+  p.v_new = static_cast<const __nv_bfloat16*>(v_new);
+  p.arena = c->k_base();
+  int grid = 0;
+  plan_decode(c, layer, c->lay.max_tiles, p, grid, c->t[layer] + 1);  // state after the append
+  if (p.n_tiles > c->lay.max_tiles)
+    return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = launch_decode(p, c->kv_map, c->pol.head_dim, grid, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
+  e = launch_decode_combine(p, c->pol.head_dim, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
+  c->t[layer] += 1;
   return ok();
 }
 
@@ -594,7 +630,7 @@ hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q,
   p.out = out;
   p.err = c->err();
   int grid = 0;
-  plan_decode(c, layer, cap_tiles, p, grid);
+  plan_decode(c, layer, cap_tiles, p, grid, c->t[layer]);
   if (p.n_tiles > cap_tiles)
     return fail(HWKV_EINVAL, "decode plan needs %d tiles > %d in the static scratch", p.n_tiles,
                 cap_tiles);

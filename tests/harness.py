@@ -82,6 +82,16 @@ class Run:
         hwkv.hwkv_decode_attn(self.cache, layer, q, self.scale, out, self.stream)
         return out
 
+    def decode_step_fused(self, layer):
+        """hwkv_decode_step: append the token at position t and attend, in one call."""
+        t = hwkv.hwkv_seq_len(self.cache, layer)
+        k = self.gen(hwkv_gen.K, layer, t, 1, self.Hkv)
+        v = self.gen(hwkv_gen.V, layer, t, 1, self.Hkv)
+        q = self.gen(hwkv_gen.Q, layer, t, 1, self.Hq).view(self.B, self.Hq, self.d)
+        out = self.torch.empty((self.B, self.Hq, self.d), dtype=self.torch.float32, device="cuda")
+        hwkv.hwkv_decode_step(self.cache, layer, q, k, v, self.scale, out, self.stream)
+        return out
+
     def oracle_rows(self, layer, b, qh, positions):
         h = qh // self.G
         O, sp = oracle.window_attention_gen(self.g, layer, b, h, [qh] * len(positions),

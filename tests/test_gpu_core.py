@@ -67,6 +67,37 @@ def test_decode_parity(d, Hq, Hkv, B, windows, prompt, steps):
         r.close()
 
 
+@pytest.mark.parametrize("d,Hq,Hkv,B,windows,prompt,steps", [
+    (64, 8, 2, 1, [0, 128], 120, 14),                 # crosses the window and wraps
+    (128, 8, 8, 2, [0, 1, 2, 63, 64, 65, 200, 4096], 60, 8),
+    (256, 24, 4, 2, [0, 1000, 257, 70], 1500, 3),
+    (128, 16, 2, 3, [0, 513], 2100, 2),
+])
+def test_fused_decode_step(d, Hq, Hkv, B, windows, prompt, steps):
+    """hwkv_decode_step equals append + decode_attn (oracle, twin cache, ring bytes)."""
+    r = Run(1, B, Hq, Hkv, d, prompt + steps, windows, seed=13, per_head_scale=True)
+    twin = Run(1, B, Hq, Hkv, d, prompt + steps, windows, seed=13, per_head_scale=True)
+    try:
+        r.fill(0, prompt, chunk=511)
+        twin.fill(0, prompt, chunk=511)
+        for i in range(steps):
+            got = r.decode_step_fused(0).cpu().numpy()
+            ref = twin.decode_step(0).cpu().numpy()
+            p = prompt + i
+            assert hwkv.hwkv_seq_len(r.cache, 0) == p + 1
+            assert_close(got, ref.astype(np.float64), "fused vs separate p%d" % p)
+            for b in range(B):
+                for qh in range(Hq):
+                    assert_close(got[b, qh], r.oracle_rows(0, b, qh, [p])[0],
+                                 "fused b%d q%d p%d" % (b, qh, p))
+            r.check_rings(0)
+            r.check_residency()
+        hwkv.hwkv_sync_check(r.cache)
+    finally:
+        r.close()
+        twin.close()
+
+
 def test_decode_multi_layer_independent_state():
     r = Run(3, 2, 12, 2, 256, 900, [0, 64, 300, 0, 0, 5], seed=2)
     try:
