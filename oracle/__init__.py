@@ -59,6 +59,20 @@ def lib():
                                              ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
                                              ctypes.c_int64]
         L.oracle_normalized_rate.restype = ctypes.c_double
+        L.oracle_cos_eval.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
+                                      ctypes.c_double]
+        L.oracle_cos_eval.restype = ctypes.c_double
+        L.oracle_conditional_similarity_bf16.argtypes = [
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p,
+            ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p, ctypes.c_int64, ctypes.c_double,
+            ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p]
+        L.oracle_conditional_similarity_bf16.restype = ctypes.c_int
+        L.oracle_select_window.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
+                                           ctypes.c_int64, ctypes.c_double]
+        L.oracle_select_window.restype = ctypes.c_int64
+        L.oracle_budget_select.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
+                                           ctypes.c_double]
+        L.oracle_budget_select.restype = ctypes.c_int64
         _lib = L
     return _lib
 
@@ -159,3 +173,46 @@ def normalized_rate(windows, C, dK, dV, bK=2, bV=2):
     """R_C(a), Eq. normalized-rate."""
     w = np.ascontiguousarray(windows, dtype=np.int64).ravel()
     return float(lib().oracle_normalized_rate(_p(w), len(w), C, dK, dV, bK, bV))
+
+
+EPS_COS = 1e-12  # App. A.2: epsilon of the stabilized cosine
+
+
+def cos_eval(u, v, eps=EPS_COS):
+    """Stabilized cosine (App. A.2, Eq. stabilized-cosine)."""
+    u = np.ascontiguousarray(u, dtype=np.float64)
+    v = np.ascontiguousarray(v, dtype=np.float64)
+    return float(lib().oracle_cos_eval(_p(u), _p(v), len(u), eps))
+
+
+def conditional_similarity_bf16(Q, pos, Kp, Vp, windows, gamma, eps=EPS_COS):
+    """Eq. conditional-similarity of one KV head: (scores [n_w], cos [R, n_w]).
+    Q [R, d] bf16 bits (rows = (position, query head)), pos [R], Kp/Vp [T, d]."""
+    Q = np.ascontiguousarray(Q, dtype=np.uint16)
+    Kp = np.ascontiguousarray(Kp, dtype=np.uint16)
+    Vp = np.ascontiguousarray(Vp, dtype=np.uint16)
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    W = np.ascontiguousarray(windows, dtype=np.int64)
+    R, d = Q.shape
+    scores = np.zeros(len(W))
+    cos = np.zeros((R, len(W)))
+    rc = lib().oracle_conditional_similarity_bf16(_p(Q), _p(pos), R, _p(Kp), _p(Vp), Kp.shape[0],
+                                                  d, _p(W), len(W), float(gamma), eps,
+                                                  _p(scores), _p(cos))
+    if rc != 0:
+        raise ValueError("oracle_conditional_similarity_bf16 failed (rc=%d)" % rc)
+    return scores, cos
+
+
+def select_window(scores, windows, C, tau):
+    """Eq. threshold-selection for one head; returns the window (0 = full)."""
+    s = np.ascontiguousarray(scores, dtype=np.float64)
+    W = np.ascontiguousarray(windows, dtype=np.int64)
+    return int(lib().oracle_select_window(_p(s), _p(W), len(W), int(C), float(tau)))
+
+
+def budget_select(beta, phi, budget):
+    """Eq. budget-selector: index g* (0-based) of the chosen record, or -1."""
+    b = np.ascontiguousarray(beta, dtype=np.float64)
+    f = np.ascontiguousarray(phi, dtype=np.float64)
+    return int(lib().oracle_budget_select(_p(b), _p(f), len(b), float(budget)))

@@ -20,7 +20,12 @@
  *                       (Sec. 3.1, Eq. nominal-storage);
  *   - normalized rate   R_C = N_C(a) / N_C(all full) (Sec. 3.1, Eq. normalized-rate);
  *   - physical residency: each head keeps only its latest r_t(w) K/V states
- *                       (Sec. 3.3); stored as a ring with slot(p) = p mod cap.
+ *                       (Sec. 3.3); stored as a ring with slot(p) = p mod cap;
+ *   - SeqCalib scoring and selection: stabilized cosine (App. A.2,
+ *                       Eq. stabilized-cosine), conditional similarity
+ *                       (Eq. conditional-similarity), threshold selection
+ *                       (Eq. threshold-selection), budget selector (App. A.2,
+ *                       Eq. budget-selector).
  *
  * Windows are int64: 0 (HWKV_WINDOW_FULL) means full history; any W >= the
  * context is equivalent to full (Sec. 3.1). bf16 inputs are widened exactly to
@@ -267,4 +272,107 @@ double oracle_normalized_rate(const int64_t* W, int64_t n_units, int64_t C, int6
   uint64_t den = 0;
   for (int64_t u = 0; u < n_units; ++u) den += (uint64_t)C * (uint64_t)(dK * bK + dV * bV);
   return den ? (double)num / (double)den : 0.0;
+}
+
+/* ------------------------------------------------------ SeqCalib (App. A.2) */
+
+/*
+ * Stabilized cosine, App. "Calibration Score and Fixed-Prefix Selection",
+ * Eq. stabilized-cosine: a vector of norm <= eps counts as zero; both zero
+ * gives 1, exactly one zero gives 0, otherwise the plain cosine.
+ */
+double oracle_cos_eval(const double* u, const double* v, int64_t d, double eps) {
+  double uu = 0.0, vv = 0.0, uv = 0.0;
+  for (int64_t i = 0; i < d; ++i) {
+    uu += u[i] * u[i];
+    vv += v[i] * v[i];
+    uv += u[i] * v[i];
+  }
+  const double nu = sqrt(uu), nv = sqrt(vv);
+  const int zu = nu <= eps, zv = nv <= eps;
+  if (zu && zv) return 1.0;
+  if (zu || zv) return 0.0;
+  return uv / (nu * nv);
+}
+
+/*
+ * Conditional similarity of one KV head (Sec. 3.2, Eq. conditional-similarity):
+ * for every candidate window W[k] (k < n_w, finite), the mean over the rows
+ * (sampled position, query head) of cos_eval(o^(W[k]), o^(full)), where o^(w)
+ * is Eq. conditional-attention over J_p(w). Rows: q row r at Q + r*d with
+ * position pos[r]; K, V [T][d] hold positions 0..T-1 of this head.
+ * scores[k] receives the means; cos_out (optional) [R][n_w] the individual scores.
+ */
+int oracle_conditional_similarity_bf16(const uint16_t* Q, const int64_t* pos, int64_t R,
+                                       const uint16_t* Kp, const uint16_t* Vp, int64_t T,
+                                       int64_t d, const int64_t* W, int64_t n_w, double gamma,
+                                       double eps, double* scores, double* cos_out) {
+  if (R <= 0 || d <= 0 || n_w < 0) return 1;
+  double* of = (double*)malloc(sizeof(double) * (size_t)(R * d));
+  double* ow = (double*)malloc(sizeof(double) * (size_t)(R * d));
+  double* c = (double*)malloc(sizeof(double) * (size_t)(R * (n_w > 0 ? n_w : 1)));
+  if (!of || !ow || !c) {
+    free(of);
+    free(ow);
+    free(c);
+    return 2;
+  }
+  int rc = oracle_window_attention_bf16(Q, d, pos, R, Kp, Vp, d, T, d, ORACLE_FULL, gamma, of, NULL);
+  for (int64_t k = 0; rc == 0 && k < n_w; ++k) {
+    rc = oracle_window_attention_bf16(Q, d, pos, R, Kp, Vp, d, T, d, W[k], gamma, ow, NULL);
+    double sum = 0.0;
+    for (int64_t r = 0; rc == 0 && r < R; ++r) {
+      c[r * n_w + k] = oracle_cos_eval(ow + r * d, of + r * d, d, eps);
+      sum += c[r * n_w + k];
+    }
+    scores[k] = sum / (double)R;
+  }
+  if (rc == 0 && cos_out) memcpy(cos_out, c, sizeof(double) * (size_t)(R * n_w));
+  free(of);
+  free(ow);
+  free(c);
+  return rc;
+}
+
+/*
+ * Threshold selection of one head (Sec. 3.2, Eq. threshold-selection): among
+ * the candidates {W[0..n_w-1] finite, full} whose score is >= tau (full always
+ * scores 1), the lowest nominal cost r_C(w) = min(w, C); equal costs go to the
+ * earlier candidate in the order <_W (finite windows increasing, then full).
+ * Returns the chosen window, 0 for full.
+ */
+int64_t oracle_select_window(const double* scores, const int64_t* W, int64_t n_w, int64_t C,
+                             double tau) {
+  int64_t best = ORACLE_FULL;
+  int64_t best_cost = C;
+  int64_t best_rank = n_w;  /* full is last in <_W */
+  for (int64_t k = 0; k < n_w; ++k) {
+    if (!(scores[k] >= tau)) continue;
+    const int64_t cost = oracle_retained_tokens(W[k], C);
+    /* rank in <_W: finite windows by value */
+    int64_t rank = 0;
+    for (int64_t j = 0; j < n_w; ++j)
+      if (W[j] < W[k]) ++rank;
+    if (cost < best_cost || (cost == best_cost && rank < best_rank)) {
+      best = W[k];
+      best_cost = cost;
+      best_rank = rank;
+    }
+  }
+  return best;
+}
+
+/*
+ * Finite-grid budget selection (App. "Finite-grid budget selection",
+ * Eq. budget-selector): among records g with beta[g] <= budget, maximise
+ * phi[g], then minimise beta[g], then take the smallest g. Returns g (0-based)
+ * or -1 when no record meets the budget.
+ */
+int64_t oracle_budget_select(const double* beta, const double* phi, int64_t G, double budget) {
+  int64_t best = -1;
+  for (int64_t g = 0; g < G; ++g) {
+    if (!(beta[g] <= budget)) continue;
+    if (best < 0 || phi[g] > phi[best] || (phi[g] == phi[best] && beta[g] < beta[best])) best = g;
+  }
+  return best;
 }
