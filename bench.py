@@ -411,6 +411,55 @@ def run_prefill(args, local):
                 tokens_per_s=B * wl.prompt / (ms * 1e-3))
 
 
+# ------------------------------------------------------------ GPU SeqCalib
+def run_calib(local, T=131072, P=256, Hkv=4, Hq=24, d=256, windows=(8192, 16384, 32768), reps=3):
+    """Candidate replay of one layer's trace: a T-token trace, P query positions
+    drawn from its final quarter, every candidate window scored against full.
+    Algorithmic bytes: each (position, KV head) reads its t + 1 keys once (4 d B)."""
+    import torch
+
+    import hwkv_gen
+    import paper_2609_02029_gb300 as hwkv
+
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    s = stream.cuda_stream
+    g = hwkv_gen.desc(7)
+    rng = np.random.default_rng(3)
+    pos = np.sort(rng.choice(np.arange(T - T // 4, T), size=P, replace=False))[None, :]
+    K = torch.empty((1, T, Hkv, d), dtype=torch.bfloat16, device=dev)
+    V = torch.empty_like(K)
+    hwkv_gen.fill_device(g, hwkv_gen.K, 0, 1, 0, T, Hkv, d, K.data_ptr(), s)
+    hwkv_gen.fill_device(g, hwkv_gen.V, 0, 1, 0, T, Hkv, d, V.data_ptr(), s)
+    Kh = K.permute(0, 2, 1, 3).contiguous()
+    Vh = V.permute(0, 2, 1, 3).contiguous()
+    del K, V
+    q = torch.empty((1, P, Hq, d), dtype=torch.bfloat16, device=dev)
+    for i in range(P):
+        hwkv_gen.fill_device(g, hwkv_gen.Q, 0, 1, int(pos[0, i]), 1, Hq, d, q[0, i].data_ptr(), s)
+    desc = hwkv.make_calib_desc(1, P, Hkv, Hq, d, T, list(windows), pos)
+    nbytes = hwkv.hwkv_calib_workspace_bytes(desc)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    scale = 1.0 / np.sqrt(d)
+    times = []
+    for rep in range(reps + 1):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        scores, _ = hwkv.hwkv_calib_scores(desc, q, Kh, Vh, scale, ws, nbytes, stream)
+        t1 = time.perf_counter()  # the call synchronizes its stream
+        if rep:
+            times.append(t1 - t0)
+    sec = float(np.median(times))
+    keys = int((pos + 1).sum()) * Hkv
+    del Kh, Vh, q, ws
+    torch.cuda.empty_cache()
+    return {"trace_tokens": T, "positions": P, "kv_heads": Hkv, "q_heads": Hq, "head_dim": d,
+            "windows": list(windows), "ms": sec * 1e3, "keys_replayed": keys,
+            "gbs": keys * 4 * d / sec / 1e9, "positions_per_s": P / sec,
+            "mean_scores": [float(x) for x in scores.mean(axis=0)],
+            "note": "wall time of hwkv_calib_scores (plan, upload, both kernels, readback)"}
+
+
 # ------------------------------------------------------------ CPU oracle
 def step_keys(wl, max_ctx, t):
     """(layer, batch row, KV head) units of one decode step at length t and the
@@ -530,6 +579,7 @@ def main():
     ap.add_argument("--prefill-reps", type=int, default=3)
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-calib", action="store_true")
     ap.add_argument("--prefill-only", action="store_true",
                     help="run only the 64K prefill measurement (profiling)")
     ap.add_argument("--layers", type=int, default=0,
@@ -598,6 +648,9 @@ def main():
     pre = None
     if not args.no_prefill and rank == 0:
         pre = run_prefill(args, local)
+    cal = None
+    if rank == 0 and not args.no_calib:
+        cal = run_calib(local)
     cb = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cb = cpu_baseline(wl, r["max_ctx"], r["t_first"] + 1)
@@ -635,6 +688,8 @@ def main():
                            "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst,
                            "peak_source": peak_src, "ms": pre["ms"],
                            "tokens_per_s": pre["tokens_per_s"], "flops": pre["flops"]}
+    if cal is not None:
+        line["seqcalib"] = cal
     if cb is not None:
         line["cpu_baseline"] = cb
     emit(line)

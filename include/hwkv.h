@@ -188,6 +188,66 @@ HWKV_API hwkv_status hwkv_decode_attn_static(hwkv_cache* cache, int32_t layer, c
                                              float scale, float* out, void* cuda_stream);
 
 /*
+ * SeqCalib candidate replay (Sec. 3.2: one layer's trace, every candidate
+ * window replayed from it). For query head q at sampled position t of
+ * calibration sequence n, o^(w) is the attention output over the keys
+ * [max(0, t-w+1), t] (Eq. conditional-attention) and
+ *   cos[n][p][q][k] = cos_eval(o^(windows[k]), o^(full))   (App. A.2,
+ *                     Eq. stabilized-cosine, eps = 1e-12),
+ *   scores[h][k]    = mean of cos over (n, p, q in the group of KV head h)
+ *                     (Eq. conditional-similarity).
+ * The full candidate scores one and is not listed.
+ */
+typedef struct {
+  int32_t n_seq;       /* calibration sequences N */
+  int32_t n_pos;       /* sampled query positions per sequence P */
+  int32_t n_kv_heads;
+  int32_t n_q_heads;   /* multiple of n_kv_heads, group <= 8 */
+  int32_t head_dim;    /* 64, 128 or 256 */
+  int32_t n_windows;   /* K candidate finite windows, 1..8 */
+  int64_t T;           /* trace length: positions 0..T-1 */
+  const int64_t* windows;    /* [K] host, positive, increasing */
+  const int64_t* positions;  /* [N][P] host, in [0, T) */
+} hwkv_calib_desc;
+
+/* Device workspace hwkv_calib_scores needs for this description (host-only). */
+HWKV_API hwkv_status hwkv_calib_workspace_bytes(const hwkv_calib_desc* desc, size_t* bytes);
+
+/*
+ *   q:    [N][P][n_q_heads][head_dim] bf16, device: queries at the sampled positions
+ *   k, v: [N][n_kv_heads][T][head_dim] bf16, device: the layer's trace, head-major
+ *   workspace: device, >= hwkv_calib_workspace_bytes(desc), 256-byte aligned
+ *   scores: host [n_kv_heads][K] double; cos_out: host [N][P][n_q_heads][K] float or NULL
+ * The keys of each (sequence, position, KV head) are cut into the nested
+ * suffix bands of the windows, replayed once with split-KV tiles, and merged
+ * band by band. Synchronizes `cuda_stream` (results are returned on the host).
+ */
+HWKV_API hwkv_status hwkv_calib_scores(const hwkv_calib_desc* desc, const void* q, const void* k,
+                                       const void* v, float scale, void* workspace,
+                                       size_t ws_bytes, double* scores, float* cos_out,
+                                       void* cuda_stream);
+
+/*
+ * Threshold selection (Sec. 3.2, Eq. threshold-selection) for each of n_heads
+ * heads: among the windows whose score is >= tau, plus full (score one), the
+ * one of lowest nominal cost min(w, C); equal costs go to the earlier window in
+ * the order <_W (increasing finite windows, then full). policy[h] receives the
+ * window, HWKV_WINDOW_FULL for full. scores: [n_heads][n_windows]. Host-only.
+ */
+HWKV_API hwkv_status hwkv_calib_select(const double* scores, int32_t n_heads,
+                                       const int64_t* windows, int32_t n_windows, int64_t C,
+                                       double tau, int64_t* policy);
+
+/*
+ * Finite-grid budget selection (App. A.2, Eq. budget-selector): among the
+ * records g with beta[g] <= budget, the largest phi[g], then the smallest
+ * beta[g], then the smallest g; *chosen = g, or -1 if no record meets the
+ * budget. Host-only.
+ */
+HWKV_API hwkv_status hwkv_budget_select(const double* beta, const double* phi, int32_t n_records,
+                                        double budget, int32_t* chosen);
+
+/*
  * Resident K+V bytes (Sec. 3.1, Eq. nominal-storage with C = t, bf16 K and V,
  * times batch): sum over KV heads of batch * min(cap, t) * head_dim * 2 * 2,
  * for one layer, or summed over all layers when layer == -1. Host-only.

@@ -47,6 +47,25 @@ def make_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, max_ctx, windo
     return pol
 
 
+class hwkv_calib_desc(ctypes.Structure):
+    _fields_ = [("n_seq", ctypes.c_int32), ("n_pos", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("n_windows", ctypes.c_int32),
+                ("T", ctypes.c_int64), ("windows", ctypes.POINTER(ctypes.c_int64)),
+                ("positions", ctypes.POINTER(ctypes.c_int64))]
+
+
+def make_calib_desc(n_seq, n_pos, n_kv_heads, n_q_heads, head_dim, T, windows, positions):
+    """hwkv_calib_desc with its windows [K] and positions [n_seq, n_pos] kept alive."""
+    w = np.ascontiguousarray(np.asarray(windows, dtype=np.int64).ravel())
+    pos = np.ascontiguousarray(np.asarray(positions, dtype=np.int64).ravel())
+    d = hwkv_calib_desc(n_seq, n_pos, n_kv_heads, n_q_heads, head_dim, len(w), T,
+                        w.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+                        pos.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)))
+    d._keepalive = (w, pos)
+    return d
+
+
 _lib = None
 _vp, _i32, _i64, _u64p = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.POINTER(ctypes.c_uint64)
 
@@ -75,6 +94,12 @@ def lib():
             "hwkv_ring_capacity": [_vp, _i32, _i32, ctypes.POINTER(_i64)],
             "hwkv_debug_copy_ring": [_vp, _i32, _i32, _i32, _vp, _vp],
             "hwkv_sync_check": [_vp],
+            "hwkv_calib_workspace_bytes": [ctypes.POINTER(hwkv_calib_desc),
+                                           ctypes.POINTER(ctypes.c_size_t)],
+            "hwkv_calib_scores": [ctypes.POINTER(hwkv_calib_desc), _vp, _vp, _vp, ctypes.c_float,
+                                  _vp, ctypes.c_size_t, _vp, _vp, _vp],
+            "hwkv_calib_select": [_vp, _i32, _vp, _i32, _i64, ctypes.c_double, _vp],
+            "hwkv_budget_select": [_vp, _vp, _i32, ctypes.c_double, ctypes.POINTER(_i32)],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -201,3 +226,40 @@ def hwkv_debug_copy_ring(cache, layer, b, kv_head, head_dim):
 
 def hwkv_sync_check(cache):
     _check(lib().hwkv_sync_check(cache))
+
+
+def hwkv_calib_workspace_bytes(desc):
+    n = ctypes.c_size_t(0)
+    _check(lib().hwkv_calib_workspace_bytes(ctypes.byref(desc), ctypes.byref(n)))
+    return n.value
+
+
+def hwkv_calib_scores(desc, q, k, v, scale, workspace, ws_bytes, stream=None, with_cos=False):
+    """(scores [n_kv_heads, K] float64, cos [N, P, n_q_heads, K] float32 or None)."""
+    K = desc.n_windows
+    scores = np.zeros((desc.n_kv_heads, K), dtype=np.float64)
+    cos = np.zeros((desc.n_seq, desc.n_pos, desc.n_q_heads, K), dtype=np.float32) if with_cos else None
+    _check(lib().hwkv_calib_scores(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), scale,
+                                   _ptr(workspace), ws_bytes, scores.ctypes.data_as(_vp),
+                                   cos.ctypes.data_as(_vp) if cos is not None else None,
+                                   _stream(stream)))
+    return scores, cos
+
+
+def hwkv_calib_select(scores, windows, C, tau):
+    s = np.ascontiguousarray(scores, dtype=np.float64)
+    w = np.ascontiguousarray(windows, dtype=np.int64)
+    H = s.shape[0]
+    out = np.zeros(H, dtype=np.int64)
+    _check(lib().hwkv_calib_select(s.ctypes.data_as(_vp), H, w.ctypes.data_as(_vp), len(w), C,
+                                   tau, out.ctypes.data_as(_vp)))
+    return out
+
+
+def hwkv_budget_select(beta, phi, budget):
+    b = np.ascontiguousarray(beta, dtype=np.float64)
+    f = np.ascontiguousarray(phi, dtype=np.float64)
+    g = ctypes.c_int32(0)
+    _check(lib().hwkv_budget_select(b.ctypes.data_as(_vp), f.ctypes.data_as(_vp), len(b), budget,
+                                    ctypes.byref(g)))
+    return g.value

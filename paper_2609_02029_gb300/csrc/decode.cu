@@ -37,6 +37,16 @@ struct TileInfo {
 
 __device__ __forceinline__ TileInfo locate_tile(const DecodeParams& p, int tile) {
   TileInfo ti;
+  if (p.tiles != nullptr) {  // explicit tile table
+    const CalibTile ct = p.tiles[tile];
+    ti.b = ct.q_row;
+    ti.h = ct.h;
+    ti.start = 0;
+    ti.len = ct.len;
+    ti.k_row = ct.k_row;
+    ti.v_row = ct.v_row;
+    return ti;
+  }
   ti.b = tile / p.tiles_per_b;
   const int lt = tile - ti.b * p.tiles_per_b;
   int h = 0;
@@ -77,7 +87,8 @@ struct DecodeCfg {
 
 template <int D>
 __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
-    decode_split_kernel(const __grid_constant__ CUtensorMap kv_map, const DecodeParams p) {
+    decode_split_kernel(const __grid_constant__ CUtensorMap k_map,
+                        const __grid_constant__ CUtensorMap v_map, const DecodeParams p) {
   using C = DecodeCfg<D>;
   constexpr int STAGES = C::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -105,7 +116,8 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
   if (warp == kDecodeWarps) {
     // ------------------------------------------------------------ producer
     if (lane != 0) return;
-    prefetch_tensormap(&kv_map);
+    prefetch_tensormap(&k_map);
+    prefetch_tensormap(&v_map);
     uint32_t it = 0;
     bool ok = true;
     for (int tile = blockIdx.x; ok && tile < p.n_tiles; tile += gridDim.x) {
@@ -125,10 +137,10 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
         const int32_t vrow = (int32_t)(ti.v_row + (int64_t)st * kStageTokens);
 #pragma unroll
         for (int sl = 0; sl < C::kSlabs; ++sl)
-          tma_load_2d(kdst + sl * kSlabBytes, &kv_map, sl * 64, krow, &full[s]);
+          tma_load_2d(kdst + sl * kSlabBytes, &k_map, sl * 64, krow, &full[s]);
 #pragma unroll
         for (int sl = 0; sl < C::kSlabs; ++sl)
-          tma_load_2d(vdst + sl * kSlabBytes, &kv_map, sl * 64, vrow, &full[s]);
+          tma_load_2d(vdst + sl * kSlabBytes, &v_map, sl * 64, vrow, &full[s]);
       }
     }
     if (!ok) {
@@ -302,7 +314,7 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     {
       // one tile covers the whole ring: this is the final output, normalised here;
       // otherwise leave the tile's partial for the combine kernel
-      const bool single = p.u[ti.h].n_tiles == 1;
+      const bool single = p.tiles == nullptr && p.u[ti.h].n_tiles == 1;
       float* po = p.part_o + (int64_t)tile * kMaxGroup * D;
       float* fo = p.out + ((int64_t)ti.b * p.n_q_heads + (int64_t)ti.h * p.group) * D;
       for (int n = 0; n < p.group; ++n) {
@@ -411,22 +423,129 @@ int decode_smem_bytes(int head_dim) {
 }
 
 template <int D>
-static cudaError_t launch_decode_t(const DecodeParams& p, const CUtensorMap& map, int grid,
-                                   cudaStream_t s) {
+static cudaError_t launch_decode_t(const DecodeParams& p, const CUtensorMap& kmap,
+                                   const CUtensorMap& vmap, int grid, cudaStream_t s) {
   const int smem = DecodeCfg<D>::kSmem;
   cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(decode_split_kernel<D>, dim3(grid), dim3((kDecodeWarps + 1) * 32), smem, s,
-                    map, p);
+                    kmap, vmap, p);
 }
 
-cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& map, int head_dim, int grid,
-                          cudaStream_t s) {
+cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& kmap, const CUtensorMap& vmap,
+                          int head_dim, int grid, cudaStream_t s) {
   switch (head_dim) {
-    case 64: return launch_decode_t<64>(p, map, grid, s);
-    case 128: return launch_decode_t<128>(p, map, grid, s);
-    case 256: return launch_decode_t<256>(p, map, grid, s);
+    case 64: return launch_decode_t<64>(p, kmap, vmap, grid, s);
+    case 128: return launch_decode_t<128>(p, kmap, vmap, grid, s);
+    case 256: return launch_decode_t<256>(p, kmap, vmap, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+// SeqCalib candidate replay (Sec. 3.2, Eq. conditional-similarity; App. A.2,
+// Eq. stabilized-cosine). For one unit (sequence, sampled position, KV head)
+// the keys were split into nested-suffix bands: band 0 = the newest W_0 keys,
+// band k = keys between W_{k-1} and W_k back, band K = everything older. Warp g
+// merges the band partials of query head g in band order; after band k (< K)
+// the running output is o^(W_k), after the last band it is o^(full). Each
+// candidate is scored against full with the stabilized cosine (eps = 1e-12:
+// a vector of norm <= eps counts as zero; both zero -> 1, one zero -> 0).
+constexpr int kCalibMaxWindows = 8;
+
+template <int D>
+__global__ void __launch_bounds__(kMaxGroup * 32) calib_combine_kernel(const CalibCombineParams p) {
+  constexpr int PER = D / 32;
+  grid_dep_wait();
+  const int u = blockIdx.x;
+  const int g = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (g >= p.group) return;
+  const int K = p.n_windows;
+  const float c = p.scale_log2;
+  const int32_t* bb = p.band_begin + (int64_t)u * (K + 2);
+  float M = -INFINITY, L = 0.f;
+  float O[PER];
+#pragma unroll
+  for (int e = 0; e < PER; ++e) O[e] = 0.f;
+  float snap[kCalibMaxWindows][PER];
+  float snap_l[kCalibMaxWindows];
+#pragma unroll
+  for (int k = 0; k < kCalibMaxWindows; ++k) {
+    snap_l[k] = 0.f;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) snap[k][e] = 0.f;
+  }
+  for (int k = 0; k <= K; ++k) {
+    for (int j = bb[k]; j < bb[k + 1]; ++j) {
+      const float2 ml = p.part_ml[(int64_t)j * kMaxGroup + g];
+      if (ml.x == -INFINITY) continue;
+      const float nm = fmaxf(M, ml.x);
+      const float a = M == -INFINITY ? 0.f : ex2((M - nm) * c);
+      const float bw = ex2((ml.x - nm) * c);
+      const float* src = p.part_o + ((int64_t)j * kMaxGroup + g) * D + lane * PER;
+#pragma unroll
+      for (int e = 0; e < PER; ++e) O[e] = O[e] * a + src[e] * bw;
+      L = L * a + ml.y * bw;
+      M = nm;
+    }
+    if (k < K) {  // o^(W_k) up to the common factor 2^{-M c}, normalised below
+#pragma unroll
+      for (int kk = 0; kk < kCalibMaxWindows; ++kk)
+        if (kk == k) {
+          snap_l[kk] = L;
+#pragma unroll
+          for (int e = 0; e < PER; ++e) snap[kk][e] = O[e];
+        }
+      // later bands rescale O by 2^{(M_old - M_new) c}; keep the snapshots' reference
+      // by storing them normalised now
+#pragma unroll
+      for (int kk = 0; kk < kCalibMaxWindows; ++kk)
+        if (kk == k) {
+          const float inv = snap_l[kk] > 0.f ? 1.f / snap_l[kk] : 0.f;
+#pragma unroll
+          for (int e = 0; e < PER; ++e) snap[kk][e] *= inv;
+        }
+    }
+  }
+  const float invL = L > 0.f ? 1.f / L : 0.f;
+  float full[PER];
+  float ff = 0.f;
+#pragma unroll
+  for (int e = 0; e < PER; ++e) {
+    full[e] = O[e] * invL;
+    ff += full[e] * full[e];
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) ff += __shfl_xor_sync(0xffffffffu, ff, off);
+  const float nf = sqrtf(ff);
+#pragma unroll
+  for (int k = 0; k < kCalibMaxWindows; ++k) {
+    if (k >= K) break;
+    float uu = 0.f, uv = 0.f;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) {
+      uu += snap[k][e] * snap[k][e];
+      uv += snap[k][e] * full[e];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      uu += __shfl_xor_sync(0xffffffffu, uu, off);
+      uv += __shfl_xor_sync(0xffffffffu, uv, off);
+    }
+    const float nu = sqrtf(uu);
+    const bool zu = nu <= 1e-12f, zf = nf <= 1e-12f;
+    const float cv = (zu && zf) ? 1.f : ((zu || zf) ? 0.f : uv / (nu * nf));
+    if (lane == 0) p.cos[((int64_t)u * p.group + g) * K + k] = cv;
+  }
+}
+
+cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cudaStream_t s) {
+  if (p.n_windows > kCalibMaxWindows || p.n_units == 0) return cudaErrorInvalidValue;
+  const dim3 grid(p.n_units), block(kMaxGroup * 32);
+  switch (head_dim) {
+    case 64: return launch_pdl(calib_combine_kernel<64>, grid, block, 0, s, p);
+    case 128: return launch_pdl(calib_combine_kernel<128>, grid, block, 0, s, p);
+    case 256: return launch_pdl(calib_combine_kernel<256>, grid, block, 0, s, p);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -36,6 +36,13 @@ struct DecodeUnit {
   int32_t s_new;       // fused step: ring slot that receives the new token
 };
 
+// a tile of explicit key rows (SeqCalib replay): rows k_row.. / v_row.. of the trace
+// maps, queries of row q_row of q, KV head h
+struct CalibTile {
+  int64_t k_row, v_row;
+  int32_t len, q_row, h, pad;
+};
+
 struct DecodeParams {
   int32_t n_units;      // KV heads of the layer
   int32_t batch;
@@ -55,7 +62,21 @@ struct DecodeParams {
   const __nv_bfloat16* k_new;  // null: plain decode over the current ring contents
   const __nv_bfloat16* v_new;
   __nv_bfloat16* arena;        // K/V rows: row r at arena + r * D
+  // table mode (SeqCalib replay): tiles[n_tiles] replace the ring plan; every tile
+  // leaves a partial (no single-tile shortcut)
+  const CalibTile* tiles;
   DecodeUnit u[kMaxKvHeads];
+};
+
+struct CalibCombineParams {
+  int32_t n_units;      // (sequence, position, KV head) units
+  int32_t group;        // G
+  int32_t n_windows;    // K candidate windows (bands K + 1)
+  float scale_log2;
+  const int32_t* band_begin;  // [n_units][K + 2]: first tile of each band, then the end
+  const float* part_o;        // [tiles][kMaxGroup][D]
+  const float2* part_ml;      // [tiles][kMaxGroup]
+  float* cos;                 // [n_units][G][K]
 };
 
 // ------------------------------------------------------------------ append
@@ -98,8 +119,9 @@ struct PrefillParams {
 
 // launchers (defined in the kernel translation units); return cudaGetLastError()
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
-cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& kv_map, int head_dim,
-                          int grid, cudaStream_t s);
+cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& k_map,
+                          const CUtensorMap& v_map, int head_dim, int grid, cudaStream_t s);
+cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cudaStream_t s);
 cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s);
 cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtensorMap& q_map,
                               const CUtensorMap& ck_map, const CUtensorMap& cv_map,

@@ -429,7 +429,7 @@ hwkv_status hwkv_decode_attn(hwkv_cache* c, int32_t layer, const void* q, float 
   if (p.n_tiles > c->lay.max_tiles)
     return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  cudaError_t e = launch_decode(p, c->kv_map, c->pol.head_dim, grid, s);
+  cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
   e = launch_decode_combine(p, c->pol.head_dim, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
@@ -465,7 +465,7 @@ hwkv_status hwkv_decode_step(hwkv_cache* c, int32_t layer, const void* q, const 
   if (p.n_tiles > c->lay.max_tiles)
     return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  cudaError_t e = launch_decode(p, c->kv_map, c->pol.head_dim, grid, s);
+  cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
   e = launch_decode_combine(p, c->pol.head_dim, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
@@ -635,10 +635,222 @@ hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q,
     return fail(HWKV_EINVAL, "decode plan needs %d tiles > %d in the static scratch", p.n_tiles,
                 cap_tiles);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  e = launch_decode(p, c->kv_map, d, grid, s);
+  e = launch_decode(p, c->kv_map, c->kv_map, d, grid, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
   e = launch_decode_combine(p, d, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
+  return ok();
+}
+
+// ---------------------------------------------------------------------------
+// SeqCalib candidate replay and selection (Sec. 3.2, Eq. conditional-similarity
+// and Eq. threshold-selection; App. A.2, Eq. stabilized-cosine and
+// Eq. budget-selector).
+
+static hwkv_status calib_validate(const hwkv_calib_desc* d) {
+  if (!d) return fail(HWKV_EINVAL, "calib desc is NULL");
+  if (d->n_seq <= 0 || d->n_pos <= 0 || d->n_kv_heads <= 0 || d->n_q_heads <= 0 || d->T <= 0)
+    return fail(HWKV_EINVAL, "calib sizes must be positive");
+  if (d->n_q_heads % d->n_kv_heads != 0) return fail(HWKV_EINVAL, "n_q_heads must be a multiple of n_kv_heads");
+  if (d->n_q_heads / d->n_kv_heads > kMaxGroup) return fail(HWKV_EUNSUPPORTED, "GQA group > 8");
+  if (d->head_dim != 64 && d->head_dim != 128 && d->head_dim != 256)
+    return fail(HWKV_EUNSUPPORTED, "head_dim %d not built", d->head_dim);
+  if (d->n_windows < 1 || d->n_windows > 8) return fail(HWKV_EUNSUPPORTED, "1..8 candidate windows");
+  if (!d->windows || !d->positions) return fail(HWKV_EINVAL, "windows/positions is NULL");
+  for (int k = 0; k < d->n_windows; ++k)
+    if (d->windows[k] <= 0 || (k > 0 && d->windows[k] <= d->windows[k - 1]))
+      return fail(HWKV_EINVAL, "candidate windows must be positive and increasing");
+  for (int64_t i = 0; i < (int64_t)d->n_seq * d->n_pos; ++i)
+    if (d->positions[i] < 0 || d->positions[i] >= d->T)
+      return fail(HWKV_EINVAL, "position %lld outside [0, T)", (long long)d->positions[i]);
+  if ((int64_t)d->n_seq * d->n_kv_heads * d->T + kStageTokens >= (int64_t)INT32_MAX)
+    return fail(HWKV_EUNSUPPORTED, "trace rows exceed the TMA coordinate range");
+  return HWKV_OK;
+}
+
+struct CalibPlan {
+  std::vector<CalibTile> tiles;
+  std::vector<int32_t> band_begin;  // [units][K + 2]
+  int64_t units = 0;
+  size_t off_tiles = 0, off_bands = 0, off_o = 0, off_ml = 0, off_cos = 0, off_err = 0, total = 0;
+};
+
+// Nested-suffix bands of position t for increasing windows W[0..K-1]: band 0 =
+// [t-W0+1, t], band k = [t-Wk+1, t-W(k-1)], band K = [0, t-W(K-1)] (clipped at 0),
+// each cut into tiles of at most tile_len keys.
+static CalibPlan calib_plan(const hwkv_calib_desc* d) {
+  CalibPlan P;
+  const int K = d->n_windows, H = d->n_kv_heads, G = d->n_q_heads / d->n_kv_heads;
+  P.units = (int64_t)d->n_seq * d->n_pos * H;
+  int64_t total_keys = 0;
+  for (int64_t i = 0; i < (int64_t)d->n_seq * d->n_pos; ++i) total_keys += (d->positions[i] + 1) * H;
+  int64_t tile_len = (total_keys / 1216 + 63) / 64 * 64;  // about 8 tiles per SM of 152
+  tile_len = std::min<int64_t>(8192, std::max<int64_t>(512, tile_len));
+  P.band_begin.reserve(P.units * (K + 2));
+  for (int n = 0; n < d->n_seq; ++n)
+    for (int pp = 0; pp < d->n_pos; ++pp)
+      for (int h = 0; h < H; ++h) {
+        const int64_t t = d->positions[(int64_t)n * d->n_pos + pp];
+        const int64_t row0 = ((int64_t)n * H + h) * d->T;
+        for (int k = 0; k <= K; ++k) {
+          const int64_t hi = k == 0 ? t : t - d->windows[k - 1];
+          const int64_t lo = k == K ? 0 : std::max<int64_t>(0, t - d->windows[k] + 1);
+          P.band_begin.push_back((int32_t)P.tiles.size());
+          for (int64_t s0 = lo; s0 <= hi; s0 += tile_len) {
+            CalibTile ct{};
+            ct.k_row = row0 + s0;
+            ct.v_row = row0 + s0;
+            ct.len = (int32_t)std::min<int64_t>(tile_len, hi - s0 + 1);
+            ct.q_row = n * d->n_pos + pp;
+            ct.h = h;
+            P.tiles.push_back(ct);
+          }
+        }
+        P.band_begin.push_back((int32_t)P.tiles.size());
+      }
+  const size_t nt = std::max<size_t>(P.tiles.size(), 1);
+  P.off_tiles = 0;
+  P.off_bands = align_up(nt * sizeof(CalibTile), kAlign);
+  P.off_o = align_up(P.off_bands + P.band_begin.size() * 4, kAlign);
+  P.off_ml = align_up(P.off_o + nt * kMaxGroup * d->head_dim * 4, kAlign);
+  P.off_cos = align_up(P.off_ml + nt * kMaxGroup * 8, kAlign);
+  P.off_err = align_up(P.off_cos + (size_t)P.units * G * K * 4, kAlign);
+  P.total = align_up(P.off_err + 64, kAlign);
+  return P;
+}
+
+hwkv_status hwkv_calib_workspace_bytes(const hwkv_calib_desc* d, size_t* bytes) {
+  if (!bytes) return fail(HWKV_EINVAL, "bytes is NULL");
+  hwkv_status st = calib_validate(d);
+  if (st != HWKV_OK) return st;
+  *bytes = calib_plan(d).total;
+  return ok();
+}
+
+hwkv_status hwkv_calib_scores(const hwkv_calib_desc* d, const void* q, const void* k,
+                              const void* v, float scale, void* workspace, size_t ws_bytes,
+                              double* scores, float* cos_out, void* cuda_stream) {
+  hwkv_status st = calib_validate(d);
+  if (st != HWKV_OK) return st;
+  if (!q || !k || !v || !workspace || !scores) return fail(HWKV_EINVAL, "NULL argument");
+  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
+  const CalibPlan P = calib_plan(d);
+  if (ws_bytes < P.total) return fail(HWKV_ENOMEM, "workspace %zu < required %zu", ws_bytes, P.total);
+  auto encode = get_encode();
+  if (!encode) return fail(HWKV_ECUDA, "cuTensorMapEncodeTiled entry point unavailable");
+  const int D = d->head_dim, H = d->n_kv_heads, G = d->n_q_heads / d->n_kv_heads, K = d->n_windows;
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  // trace maps: head-major [n_seq][n_kv_heads][T][D] seen as rows of D bf16
+  CUtensorMap kmap, vmap;
+  const cuuint64_t gdim[2] = {(cuuint64_t)D, (cuuint64_t)d->n_seq * H * d->T};
+  const cuuint64_t gstr[1] = {(cuuint64_t)D * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kStageTokens};
+  const cuuint32_t est[2] = {1, 1};
+  CUresult r = encode(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(k), gdim, gstr,
+                      box, est, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r == CUDA_SUCCESS)
+    r = encode(&vmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(v), gdim, gstr, box,
+               est, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(HWKV_EINVAL, "trace tensor map rejected (%d): k/v must be 16-byte aligned", (int)r);
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess && !P.tiles.empty())
+    e = cudaMemcpyAsync(ws + P.off_tiles, P.tiles.data(), P.tiles.size() * sizeof(CalibTile),
+                        cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(ws + P.off_bands, P.band_begin.data(), P.band_begin.size() * 4,
+                        cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ws + P.off_err, 0, 64, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "calib setup: %s", cudaGetErrorString(e));
+  DecodeParams p{};
+  p.n_units = H;
+  p.batch = 1;
+  p.group = G;
+  p.n_q_heads = d->n_q_heads;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.part_o = reinterpret_cast<float*>(ws + P.off_o);
+  p.part_ml = reinterpret_cast<float2*>(ws + P.off_ml);
+  p.err = reinterpret_cast<int*>(ws + P.off_err);
+  p.tiles = reinterpret_cast<const CalibTile*>(ws + P.off_tiles);
+  p.n_tiles = (int32_t)P.tiles.size();
+  p.tiles_per_b = p.n_tiles;
+  if (p.n_tiles > 0) {
+    e = launch_decode(p, kmap, vmap, D, std::min(p.n_tiles, std::max(1, sms)), s);
+    if (e != cudaSuccess) return fail(HWKV_ECUDA, "calib tile launch: %s", cudaGetErrorString(e));
+  }
+  CalibCombineParams cp{};
+  cp.n_units = (int32_t)P.units;
+  cp.group = G;
+  cp.n_windows = K;
+  cp.scale_log2 = p.scale_log2;
+  cp.band_begin = reinterpret_cast<const int32_t*>(ws + P.off_bands);
+  cp.part_o = p.part_o;
+  cp.part_ml = p.part_ml;
+  cp.cos = reinterpret_cast<float*>(ws + P.off_cos);
+  e = launch_calib_combine(cp, D, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "calib combine launch: %s", cudaGetErrorString(e));
+  std::vector<float> cosv((size_t)P.units * G * K);
+  int err_word = 0;
+  e = cudaMemcpyAsync(cosv.data(), cp.cos, cosv.size() * 4, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&err_word, p.err, sizeof(int), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "calib readback: %s", cudaGetErrorString(e));
+  if (err_word != 0) return fail(HWKV_EKERNEL, "calib kernel error word 0x%x", err_word);
+  // Eq. conditional-similarity: mean over (sequence, position, query head), fixed order
+  const double inv = 1.0 / ((double)d->n_seq * d->n_pos * G);
+  for (int h = 0; h < H; ++h)
+    for (int kk = 0; kk < K; ++kk) {
+      double acc = 0.0;
+      for (int64_t np = 0; np < (int64_t)d->n_seq * d->n_pos; ++np)
+        for (int g = 0; g < G; ++g) acc += cosv[((np * H + h) * G + g) * K + kk];
+      scores[h * K + kk] = acc * inv;
+    }
+  if (cos_out)  // [n_seq][n_pos][n_q_heads][K]
+    for (int64_t np = 0; np < (int64_t)d->n_seq * d->n_pos; ++np)
+      for (int h = 0; h < H; ++h)
+        for (int g = 0; g < G; ++g)
+          for (int kk = 0; kk < K; ++kk)
+            cos_out[((np * d->n_q_heads) + h * G + g) * K + kk] = cosv[((np * H + h) * G + g) * K + kk];
+  return ok();
+}
+
+hwkv_status hwkv_calib_select(const double* scores, int32_t n_heads, const int64_t* windows,
+                              int32_t n_windows, int64_t C, double tau, int64_t* policy) {
+  if (!scores || !windows || !policy || n_heads <= 0 || n_windows < 0 || C <= 0)
+    return fail(HWKV_EINVAL, "bad selection arguments");
+  for (int k = 1; k < n_windows; ++k)
+    if (windows[k] <= windows[k - 1]) return fail(HWKV_EINVAL, "windows must be increasing");
+  for (int h = 0; h < n_heads; ++h) {
+    // candidates in <_W order: finite windows increasing, then full (score one)
+    int64_t pick = HWKV_WINDOW_FULL, pick_cost = C;
+    for (int k = n_windows - 1; k >= 0; --k) {  // scan backwards: the earliest minimum wins
+      if (!(scores[(int64_t)h * n_windows + k] >= tau)) continue;
+      const int64_t cost = std::min(windows[k], C);
+      if (cost <= pick_cost) {
+        pick = windows[k];
+        pick_cost = cost;
+      }
+    }
+    policy[h] = pick;
+  }
+  return ok();
+}
+
+hwkv_status hwkv_budget_select(const double* beta, const double* phi, int32_t n_records,
+                               double budget, int32_t* chosen) {
+  if (!beta || !phi || !chosen || n_records < 0) return fail(HWKV_EINVAL, "bad selector arguments");
+  int32_t best = -1;
+  for (int32_t g = 0; g < n_records; ++g) {
+    if (!(beta[g] <= budget)) continue;
+    const bool better = best < 0 || phi[g] > phi[best] || (phi[g] == phi[best] && beta[g] < beta[best]);
+    if (better) best = g;
+  }
+  *chosen = best;
   return ok();
 }
 
