@@ -32,8 +32,10 @@ namespace hwkv {
 
 namespace {
 
-template <int D, int BN, int STAGES, int SPLIT>
+template <int D, int BN, int STAGES, int SPLIT, int SBUF = 2, int CTAS = 1>
 struct TcCfg {
+  static constexpr int kSBuf = SBUF;          // S buffers in TMEM
+  static constexpr int kCtasPerSm = CTAS;     // resident CTAs per SM (registers, TMEM, smem)
   static constexpr int kSoftmaxWarps = 4 * SPLIT;  // SPLIT warps share each TMEM lane quarter
   static constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
   static constexpr int kCW = BN / SPLIT;           // S columns per softmax warp
@@ -46,14 +48,15 @@ struct TcCfg {
   static constexpr int kTileBytes = kSlabs * kKVSlab;  // one K (or V) tile
   static constexpr int kStageBytes = 2 * kTileBytes;
   // TMEM columns: S0 [0, BN), S1 [BN, 2BN), O [2BN, 2BN + D), P [2BN + D, 2BN + D + BN/2)
-  static constexpr int kColO = 2 * BN;
-  static constexpr int kColP = 2 * BN + D;
+  static constexpr int kColO = SBUF * BN;
+  static constexpr int kColP = SBUF * BN + D;
   static constexpr int kBarBytes = 256;
   static constexpr int kRedBytes = SPLIT > 1 ? 2 * 2 * 128 * 4 : 0;  // row-max exchange
   static constexpr int kSmem =
       kQBytes + STAGES * kStageBytes + kBarBytes + kRedBytes + 1024;
-  static constexpr uint32_t kTmemCols = 512;
-  static_assert(2 * BN + D + BN / 2 <= 512, "TMEM: two S buffers, O and P");
+  static constexpr int kTmemNeed = SBUF * BN + D + BN / 2;
+  static constexpr uint32_t kTmemCols = kTmemNeed <= 128 ? 128 : (kTmemNeed <= 256 ? 256 : 512);
+  static_assert(kTmemCols * CTAS <= 512, "TMEM: S buffers, O and P of every resident CTA");
 };
 
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int32_t x,
@@ -153,13 +156,13 @@ __device__ __forceinline__ bool warp_wait_or_abort(uint64_t* bar, uint32_t parit
 
 }  // namespace
 
-template <int D, int BN, int STAGES, int SPLIT>
-__global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
+template <int D, int BN, int STAGES, int SPLIT, int SBUF, int CTAS>
+__global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThreads, CTAS)
     prefill_tc_kernel(const __grid_constant__ CUtensorMap q_map,
                       const __grid_constant__ CUtensorMap ck_map,
                       const __grid_constant__ CUtensorMap cv_map,
                       const __grid_constant__ CUtensorMap ring_map, const PrefillParams p) {
-  using C = TcCfg<D, BN, STAGES, SPLIT>;
+  using C = TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -295,9 +298,9 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
       int64_t j0;
       while (seq.next(hist, j0)) {
         const int s = j % STAGES;
-        const int sb = j & 1;
+        const int sb = j % SBUF;
         bool ok = wait_or_abort(&kv_full[s], (j / STAGES) & 1u, p.err, aborted);
-        ok = ok && wait_or_abort(&s_free[sb], ((j >> 1) & 1u) ^ 1u, p.err, aborted);
+        ok = ok && wait_or_abort(&s_free[sb], ((j / SBUF) & 1u) ^ 1u, p.err, aborted);
         if (ok) {
           tc_fence_after();
           const uint32_t k_base = smem_u32(sStage + s * C::kStageBytes);
@@ -339,7 +342,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
     int64_t j0;
     auto clampi = [](int64_t v) -> int { return (int)(v < -1 ? -1 : (v > BN + 1 ? BN + 1 : v)); };
     while (seq.next(hist, j0)) {
-      const int sb = j & 1;
+      const int sb = j % SBUF;
       // columns e of this tile visible to row pr: [a0, b0) U [a1, b1)
       int a0 = 0, b0 = 0, a1 = 0, b1 = 0;
       if (row_ok) {
@@ -360,7 +363,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
       }
       const bool full_vis = (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);
       const bool warp_full = __all_sync(0xffffffffu, full_vis);  // warp-uniform fast path
-      if (warp_wait_or_abort(&s_full[sb], (j >> 1) & 1u, p.err, aborted)) tc_fence_after();
+      if (warp_wait_or_abort(&s_full[sb], (j / SBUF) & 1u, p.err, aborted)) tc_fence_after();
       // this warp's S columns, read once into registers; the S buffer is then free
       // for the QK^T of tile j + 2 while this tile's softmax runs
       uint32_t sv[C::kCW];
@@ -485,16 +488,16 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT>::kThreads, 1)
   if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
 }
 
-template <int D, int BN, int STAGES, int SPLIT>
+template <int D, int BN, int STAGES, int SPLIT, int SBUF = 2, int CTAS = 1>
 static cudaError_t launch_tc(const PrefillParams& p, const CUtensorMap& qm, const CUtensorMap& km,
                              const CUtensorMap& vm, const CUtensorMap& rm, cudaStream_t s) {
-  using C = TcCfg<D, BN, STAGES, SPLIT>;
-  cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D, BN, STAGES, SPLIT>,
+  using C = TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>;
+  cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D, BN, STAGES, SPLIT, SBUF, CTAS>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
   if (e != cudaSuccess) return e;
   const int QP = 128 / p.group;
   dim3 grid((unsigned)((p.n + QP - 1) / QP), (unsigned)p.n_units, (unsigned)p.batch);
-  prefill_tc_kernel<D, BN, STAGES, SPLIT><<<grid, C::kThreads, C::kSmem, s>>>(qm, km, vm, rm, p);
+  prefill_tc_kernel<D, BN, STAGES, SPLIT, SBUF, CTAS><<<grid, C::kThreads, C::kSmem, s>>>(qm, km, vm, rm, p);
   return cudaGetLastError();
 }
 
@@ -505,8 +508,8 @@ cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtens
                               const CUtensorMap& ring_map, cudaStream_t s) {
   if (p.n == 0) return cudaSuccess;
   switch (head_dim) {
-    case 64: return launch_tc<64, 128, 3, 2>(p, q_map, ck_map, cv_map, ring_map, s);
-    case 128: return launch_tc<128, 128, 2, 2>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 64: return launch_tc<64, 64, 3, 1, 1, 2>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 128: return launch_tc<128, 64, 2, 1, 1, 2>(p, q_map, ck_map, cv_map, ring_map, s);
     case 256: return launch_tc<256, 64, 2, 1>(p, q_map, ck_map, cv_map, ring_map, s);
     default: return cudaErrorInvalidValue;
   }
