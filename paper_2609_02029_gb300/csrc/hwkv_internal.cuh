@@ -303,6 +303,23 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// packed fp32 pairs (sm_100+): d = a * b + c and d = a + b on two lanes at once
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)),
+        "l"(*reinterpret_cast<uint64_t*>(&c)));
+  return *reinterpret_cast<float2*>(&d);
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)));
+  return *reinterpret_cast<float2*>(&d);
+}
+
 // (lo, hi) -> bf16x2 with lo in the low half, round to nearest even
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   uint32_t r;

@@ -409,14 +409,21 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
       }
       const float bias = m_used == -INFINITY ? 0.f : m_used;
 
-      // weights 2^(z c - m), computed in place (masked logits are -inf: weight 0)
-      float s4[4] = {0.f, 0.f, 0.f, 0.f};
+      // weights 2^(z c - m), computed in place (masked logits are -inf: weight 0);
+      // the exponent arguments and the row sum in packed fp32 pairs
+      float2 s2a = make_float2(0.f, 0.f), s2b = make_float2(0.f, 0.f);
+      {
+        const float2 c2 = make_float2(c, c), nb2 = make_float2(-bias, -bias);
 #pragma unroll
-      for (int e = 0; e < C::kCW; ++e) {
-        const float w = ex2(fmaf(__uint_as_float(sv[e]), c, -bias));
-        s4[e & 3] += w;
-        sv[e] = __float_as_uint(w);
+        for (int e = 0; e < C::kCW; e += 2) {
+          const float2 y = fma2(make_float2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), c2, nb2);
+          const float2 w = make_float2(ex2(y.x), ex2(y.y));
+          if (e & 2) s2b = add2(s2b, w); else s2a = add2(s2a, w);
+          sv[e] = __float_as_uint(w.x);
+          sv[e + 1] = __float_as_uint(w.y);
+        }
       }
+      float s4[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
       const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
 
       // PV of the previous tile has read P and added into O: only now may P be
