@@ -248,6 +248,29 @@ HWKV_API hwkv_status hwkv_budget_select(const double* beta, const double* phi, i
                                         double budget, int32_t* chosen);
 
 /*
+ * Policy artifact (App. "Experimental Protocol": each calibration run stores its
+ * artifact identifier, seed and final policy matrix; App. "Runtime Realization":
+ * the runtime loads the layer x KV-head matrix once). Text format, one item per
+ * line, '#' starts a comment:
+ *   hwkv-policy 1
+ *   artifact <id: 1..127 printable characters, no spaces>
+ *   seed <unsigned 64-bit>
+ *   shape <n_layers> <n_kv_heads>
+ *   layer <l> <W_l0> <W_l1> ... <W_l(n_kv_heads-1)>     (one line per layer, in
+ *                                                      order; 0 = full)
+ * hwkv_policy_save writes `windows` [n_layers * n_kv_heads] to `path`.
+ * hwkv_policy_load reads it: windows_out must hold capacity entries; the shape
+ * and seed are returned, the id copied into artifact (NUL-terminated, artifact_cap
+ * bytes). Malformed files, negative windows or a shape larger than capacity give
+ * HWKV_EINVAL with the line number in hwkv_last_error(). Host-only.
+ */
+HWKV_API hwkv_status hwkv_policy_save(const char* path, const char* artifact, uint64_t seed,
+                                      int32_t n_layers, int32_t n_kv_heads, const int64_t* windows);
+HWKV_API hwkv_status hwkv_policy_load(const char* path, char* artifact, size_t artifact_cap,
+                                      uint64_t* seed, int32_t* n_layers, int32_t* n_kv_heads,
+                                      int64_t* windows_out, size_t capacity);
+
+/*
  * Resident K+V bytes (Sec. 3.1, Eq. nominal-storage with C = t, bf16 K and V,
  * times batch): sum over KV heads of batch * min(cap, t) * head_dim * 2 * 2,
  * for one layer, or summed over all layers when layer == -1. Host-only.

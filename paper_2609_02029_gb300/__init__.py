@@ -100,6 +100,10 @@ def lib():
                                   _vp, ctypes.c_size_t, _vp, _vp, _vp],
             "hwkv_calib_select": [_vp, _i32, _vp, _i32, _i64, ctypes.c_double, _vp],
             "hwkv_budget_select": [_vp, _vp, _i32, ctypes.c_double, ctypes.POINTER(_i32)],
+            "hwkv_policy_save": [ctypes.c_char_p, ctypes.c_char_p, ctypes.c_uint64, _i32, _i32, _vp],
+            "hwkv_policy_load": [ctypes.c_char_p, ctypes.c_char_p, ctypes.c_size_t,
+                                 ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(_i32),
+                                 ctypes.POINTER(_i32), _vp, ctypes.c_size_t],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -263,3 +267,22 @@ def hwkv_budget_select(beta, phi, budget):
     _check(lib().hwkv_budget_select(b.ctypes.data_as(_vp), f.ctypes.data_as(_vp), len(b), budget,
                                     ctypes.byref(g)))
     return g.value
+
+
+def hwkv_policy_save(path, artifact, seed, windows):
+    """Write a [n_layers, n_kv_heads] window matrix (0 = full) as a policy artifact."""
+    w = np.ascontiguousarray(np.asarray(windows, dtype=np.int64))
+    L, H = w.shape
+    _check(lib().hwkv_policy_save(str(path).encode(), artifact.encode(), seed, L, H,
+                                  w.ctypes.data_as(_vp)))
+
+
+def hwkv_policy_load(path, capacity=1 << 16):
+    """(artifact id, seed, windows [n_layers, n_kv_heads] int64)."""
+    art = ctypes.create_string_buffer(128)
+    seed = ctypes.c_uint64(0)
+    L, H = ctypes.c_int32(0), ctypes.c_int32(0)
+    out = np.zeros(capacity, dtype=np.int64)
+    _check(lib().hwkv_policy_load(str(path).encode(), art, 128, ctypes.byref(seed), ctypes.byref(L),
+                                  ctypes.byref(H), out.ctypes.data_as(_vp), capacity))
+    return art.value.decode(), seed.value, out[:L.value * H.value].reshape(L.value, H.value).copy()

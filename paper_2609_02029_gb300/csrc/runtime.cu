@@ -8,6 +8,7 @@
 // (one window level) are adjacent in one arena, K region first, then the V
 // region in the same order, then the decode workspace.
 #include <algorithm>
+#include <cerrno>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -851,6 +852,125 @@ hwkv_status hwkv_budget_select(const double* beta, const double* phi, int32_t n_
     if (better) best = g;
   }
   *chosen = best;
+  return ok();
+}
+
+// ---------------------------------------------------------------------------
+// Policy artifact I/O (App. "Experimental Protocol" / "Runtime Realization").
+
+static bool artifact_id_ok(const char* a) {
+  if (!a) return false;
+  size_t n = strlen(a);
+  if (n == 0 || n > 127) return false;
+  for (size_t i = 0; i < n; ++i)
+    if (a[i] <= ' ' || a[i] > '~') return false;
+  return true;
+}
+
+hwkv_status hwkv_policy_save(const char* path, const char* artifact, uint64_t seed,
+                             int32_t n_layers, int32_t n_kv_heads, const int64_t* windows) {
+  if (!path || !windows || n_layers <= 0 || n_kv_heads <= 0)
+    return fail(HWKV_EINVAL, "bad policy save arguments");
+  if (!artifact_id_ok(artifact))
+    return fail(HWKV_EINVAL, "artifact id must be 1..127 printable characters without spaces");
+  for (int64_t i = 0; i < (int64_t)n_layers * n_kv_heads; ++i)
+    if (windows[i] < 0) return fail(HWKV_EINVAL, "negative window at entry %lld", (long long)i);
+  FILE* f = fopen(path, "w");
+  if (!f) return fail(HWKV_EINVAL, "cannot open %s for writing", path);
+  fprintf(f, "hwkv-policy 1\nartifact %s\nseed %llu\nshape %d %d\n", artifact,
+          (unsigned long long)seed, n_layers, n_kv_heads);
+  for (int l = 0; l < n_layers; ++l) {
+    fprintf(f, "layer %d", l);
+    for (int h = 0; h < n_kv_heads; ++h) fprintf(f, " %lld", (long long)windows[(int64_t)l * n_kv_heads + h]);
+    fputc('\n', f);
+  }
+  const bool bad = ferror(f) != 0;
+  if (fclose(f) != 0 || bad) return fail(HWKV_EINVAL, "write to %s failed", path);
+  return ok();
+}
+
+hwkv_status hwkv_policy_load(const char* path, char* artifact, size_t artifact_cap, uint64_t* seed,
+                             int32_t* n_layers, int32_t* n_kv_heads, int64_t* windows_out,
+                             size_t capacity) {
+  if (!path || !artifact || artifact_cap == 0 || !seed || !n_layers || !n_kv_heads || !windows_out)
+    return fail(HWKV_EINVAL, "bad policy load arguments");
+  FILE* f = fopen(path, "r");
+  if (!f) return fail(HWKV_EINVAL, "cannot open %s", path);
+  char line[1 << 16];
+  int lineno = 0, stage = 0, next_layer = 0;
+  int32_t L = 0, H = 0;
+  hwkv_status st = HWKV_OK;
+  auto bad = [&](const char* what) {
+    st = fail(HWKV_EINVAL, "%s:%d: %s", path, lineno, what);
+    return false;
+  };
+  while (st == HWKV_OK && fgets(line, sizeof line, f)) {
+    ++lineno;
+    if (!strchr(line, '\n') && !feof(f)) { bad("line too long"); break; }
+    char* hash = strchr(line, '#');
+    if (hash) *hash = '\0';
+    char* tok = strtok(line, " \t\r\n");
+    if (!tok) continue;  // blank or comment-only line
+    const bool header = stage < 4;
+    if (stage == 0) {
+      char* v = strtok(nullptr, " \t\r\n");
+      if (strcmp(tok, "hwkv-policy") != 0 || !v || strcmp(v, "1") != 0) { bad("expected 'hwkv-policy 1'"); break; }
+      stage = 1;
+    } else if (stage == 1) {
+      char* v = strtok(nullptr, " \t\r\n");
+      if (strcmp(tok, "artifact") != 0 || !v || !artifact_id_ok(v) || strlen(v) + 1 > artifact_cap) {
+        bad("expected 'artifact <id>' fitting the buffer");
+        break;
+      }
+      strcpy(artifact, v);
+      stage = 2;
+    } else if (stage == 2) {
+      char* v = strtok(nullptr, " \t\r\n");
+      char* end = nullptr;
+      if (strcmp(tok, "seed") != 0 || !v || v[0] == '-') { bad("expected 'seed <n>'"); break; }
+      errno = 0;
+      unsigned long long sv = strtoull(v, &end, 10);
+      if (errno != 0 || !end || *end != '\0') { bad("bad seed"); break; }
+      *seed = (uint64_t)sv;
+      stage = 3;
+    } else if (stage == 3) {
+      char* a = strtok(nullptr, " \t\r\n");
+      char* b = strtok(nullptr, " \t\r\n");
+      char *ea = nullptr, *eb = nullptr;
+      long la = a ? strtol(a, &ea, 10) : 0, lb = b ? strtol(b, &eb, 10) : 0;
+      if (strcmp(tok, "shape") != 0 || !a || !b || *ea || *eb || la <= 0 || lb <= 0 ||
+          la > 4096 || lb > 4096) { bad("expected 'shape <n_layers> <n_kv_heads>'"); break; }
+      L = (int32_t)la;
+      H = (int32_t)lb;
+      if ((size_t)L * (size_t)H > capacity) { bad("policy larger than the output capacity"); break; }
+      stage = 4;
+    } else {
+      char* ls = strtok(nullptr, " \t\r\n");
+      char* e = nullptr;
+      long li = ls ? strtol(ls, &e, 10) : -1;
+      if (strcmp(tok, "layer") != 0 || !ls || *e || li != next_layer || next_layer >= L) {
+        bad("expected the next 'layer <l> ...' line");
+        break;
+      }
+      for (int h = 0; h < H; ++h) {
+        char* w = strtok(nullptr, " \t\r\n");
+        char* ew = nullptr;
+        errno = 0;
+        long long wv = w ? strtoll(w, &ew, 10) : -1;
+        if (!w || *ew || errno != 0 || wv < 0) { bad("expected a non-negative window per KV head"); break; }
+        windows_out[(size_t)next_layer * H + h] = (int64_t)wv;
+      }
+      if (st != HWKV_OK) break;
+      if (strtok(nullptr, " \t\r\n")) { bad("more windows than KV heads"); break; }
+      ++next_layer;
+    }
+    if (header && strtok(nullptr, " \t\r\n")) { bad("unexpected extra field"); break; }
+  }
+  fclose(f);
+  if (st != HWKV_OK) return st;
+  if (stage < 4 || next_layer != L) return fail(HWKV_EINVAL, "%s: incomplete policy (%d of %d layers)", path, next_layer, L);
+  *n_layers = L;
+  *n_kv_heads = H;
   return ok();
 }
 
