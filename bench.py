@@ -38,7 +38,7 @@ L2_BYTES = 129 * 1024 * 1024
 # capture (--set full) of the 1-layer, batch-2 case of layers16_112k;
 # traffic is reads of every resident K/V row plus tile partials, so it scales with the
 # algorithmic bytes of a launch. Set to None whenever that kernel changes.
-DECODE_TRAFFIC_PER_BYTE = (244.238336e6 + 3.453184e6) / 244066304.0
+DECODE_TRAFFIC_PER_BYTE = (244.297472e6 + 4.015104e6) / 244066304.0
 
 
 def peaks():
@@ -180,7 +180,8 @@ def run_gpu(args, wl, world, rank, local):
     g = hwkv_gen.desc(wl.seed + 1000003 * rank, wl.per_head_scale)  # each rank its own batch
     L, B, Hq, Hkv, d = wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim
     e2e_steps = min(args.steps, args.e2e_steps)
-    total_steps = args.warmup + args.steps + 2 + e2e_steps
+    graph_steps = min(args.steps, 32)
+    total_steps = args.warmup + args.steps + 2 + e2e_steps + 3 + graph_steps
     prompt = wl.prompt
     max_ctx = prompt + max(wl.decode_steps, total_steps)
     scale = 1.0 / np.sqrt(d)
@@ -329,7 +330,44 @@ def run_gpu(args, wl, world, rank, local):
     e2e_value = sum_over_ranks(float(B * e2e_steps), world) / (e2e_ms * 1e-3)
     h2d = int(sum(x.numel() * x.element_size() for x in host_inputs[0]))
     d2h = int(o_h.numel() * 4)
-    t_end = hwkv.hwkv_seq_len(cache, 0)
+
+    # ---- the same step as one captured CUDA graph of hwkv_decode_step_graph calls
+    # (device-side lengths and tile plan), replayed; inputs refilled between replays
+    pos = hwkv.hwkv_seq_len(cache, 0)
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        cs = torch.cuda.current_stream().cuda_stream
+        for layer in range(L):
+            hwkv.hwkv_decode_step_graph(cache, layer, q_d[layer], k_d[layer], v_d[layer], scale,
+                                        out[layer], cs)
+
+    def graph_inputs(p):
+        for layer in range(L):
+            hwkv_gen.fill_device(g, hwkv_gen.Q, layer, B, p, 1, Hq, d, q_d[layer].data_ptr(), s)
+            hwkv_gen.fill_device(g, hwkv_gen.K, layer, B, p, 1, Hkv, d, k_d[layer].data_ptr(), s)
+            hwkv_gen.fill_device(g, hwkv_gen.V, layer, B, p, 1, Hkv, d, v_d[layer].data_ptr(), s)
+
+    for i in range(3):
+        graph_inputs(pos)
+        graph.replay()
+        pos += 1
+    g_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(graph_steps)]
+    for i in range(graph_steps):
+        graph_inputs(pos)
+        if flush:
+            torch.sum(scrub, dim=0, out=scrub_out)
+        g_ev[i][0].record(stream)
+        graph.replay()
+        g_ev[i][1].record(stream)
+        pos += 1
+    g_ev[-1][1].synchronize()
+    graph_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in g_ev), world)
+    graph_value = sum_over_ranks(float(B * graph_steps), world) / (graph_ms * 1e-3)
+    del graph
+    t_end = hwkv.hwkv_seq_len(cache, 0)  # re-read from the device (graph-owned layers)
+    assert t_end == pos, (t_end, pos)
     resid_bytes = hwkv.hwkv_residency_bytes(cache, -1)
     hwkv.hwkv_sync_check(cache)
     hwkv.hwkv_free(cache)
@@ -340,7 +378,8 @@ def run_gpu(args, wl, world, rank, local):
                 dec_avg_ms=dec_avg_ms, app_avg_ms=float(np.mean(app_ms)), bytes_avg=bytes_avg,
                 achieved_gbs=achieved_gbs, step_bytes=step_bytes, clocks=clocks,
                 t_first=t_first, t_end=t_end, resid_bytes=resid_bytes,
-                launches=args.steps * L * 2, e2e_steps=e2e_steps, max_ctx=max_ctx, flush=flush)
+                launches=args.steps * L * 2, e2e_steps=e2e_steps, max_ctx=max_ctx, flush=flush,
+                graph_value=graph_value, graph_ms=graph_ms, graph_steps=graph_steps)
 
 
 # ------------------------------------------------------------- GPU prefill
@@ -682,6 +721,11 @@ def main():
                 "d2h_bytes_per_step": r["d2h"], "steps": r["e2e_steps"]},
         "gpu_launches": r["launches"],
         "clocks": r["clocks"],
+        "graph_step": {"value": r["graph_value"], "unit": "tokens/s",
+                       "ms_per_step": r["graph_ms"] / r["graph_steps"], "steps": r["graph_steps"],
+                       "note": "the same step as one CUDA graph of %d hwkv_decode_step_graph "
+                               "calls (lengths and tile plan on the device), replayed"
+                               % wl.n_layers},
     }
     if pre is not None:
         line["prefill"] = {"workload": "prefill64k", "tflops": pre["tflops"],

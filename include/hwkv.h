@@ -135,10 +135,12 @@ HWKV_API hwkv_status hwkv_prefill(hwkv_cache* cache, int32_t layer, const void* 
  * Decode attention (Sec. 3.2 at the newest position; Sec. 3.3 graph routing):
  * the query at position p = t-1 (the token the caller appended last) of each
  * query head attends over every resident slot of its KV head's ring, i.e.
- * positions [max(0, t-W), t-1], with logits scale * q.k. Work is split over
- * the rings in equal-length tiles (split count per head follows its resident
- * length), each tile yields partial (max, sum, output) and a log-sum-exp merge
- * combines them.
+ * positions [max(0, t-W), t-1], with logits scale * q.k. The kernels read
+ * the row lengths on the GPU and give every CTA an equal share of the layer's
+ * resident keys (in 64-key stages, plus a fixed cost per ring piece), so a
+ * full-history ring is split over many CTAs and short-window rings are read
+ * whole; a ring split over CTAs leaves partials (max, sum, output) that a
+ * log-sum-exp merge combines.
  *   q:   [batch, n_q_heads, head_dim] bf16
  *   out: [batch, n_q_heads, head_dim] fp32
  * Fails with HWKV_EINVAL if the layer holds no tokens.
@@ -161,6 +163,72 @@ HWKV_API hwkv_status hwkv_decode_step(hwkv_cache* cache, int32_t layer, const vo
                                       const void* k_new, const void* v_new, float scale,
                                       float* out, void* cuda_stream);
 
+/*
+ * Per-row lengths (serving form of the same method; the paper's runs decode one
+ * request at a time, so it defines no batching). Every (layer, batch row) holds
+ * its own length t_b: rows are independent sequences, and every operation above
+ * applies to each row at that row's own t_b. A row can also be idle (t_b = -1):
+ * it holds nothing, takes no append, and decode writes zeros for it. The cache
+ * keeps the lengths twice: on the host (read by the calls above) and in an
+ * int32 [n_layers][batch] array inside the arena (read by the kernels). Every
+ * call keeps both equal, except hwkv_decode_step_graph, which advances only the
+ * device copy.
+ *
+ * Decode over ragged or idle rows: hwkv_decode_attn / hwkv_decode_step accept
+ * them (the work is always planned on the GPU from the device lengths). Rows
+ * with t_b = 0 give zeros in hwkv_decode_attn.
+ */
+
+/* hwkv_append for the rows [row0, row0 + n_rows) only; each appends at its own t_b.
+ *   k, v: [n_rows, n, n_kv_heads, head_dim] bf16, device.
+ * Fails with HWKV_EINVAL for an idle row, HWKV_ECAPACITY if a row's t_b + n > max_ctx. */
+HWKV_API hwkv_status hwkv_append_rows(hwkv_cache* cache, int32_t layer, int32_t row0,
+                                      int32_t n_rows, const void* k, const void* v, int64_t n,
+                                      void* cuda_stream);
+
+/* hwkv_prefill for the rows [row0, row0 + n_rows) only (e.g. a newly admitted
+ * request); q, k, v and out hold n_rows rows. The rows must hold the same length
+ * (HWKV_EINVAL otherwise). Other errors as hwkv_prefill. */
+HWKV_API hwkv_status hwkv_prefill_rows(hwkv_cache* cache, int32_t layer, int32_t row0,
+                                       int32_t n_rows, const void* q, const void* k,
+                                       const void* v, int64_t n, float scale, float* out,
+                                       void* cuda_stream);
+
+/*
+ * hwkv_decode_step for CUDA-graph capture and replay: the step of every active
+ * row b reads t_b from the device length array at run time, appends the new
+ * token at slot t_b mod cap, attends over min(t_b + 1, cap) slots, and then
+ * advances the device t_b by one. Nothing on the host depends on the lengths,
+ * so a captured sequence of these calls (one per layer) replays as later decode
+ * steps. Idle rows get zero output and stay idle. A row already at max_ctx is
+ * skipped (zero output, length kept) and sets the error word (hwkv_sync_check).
+ * From the first such call on, the device owns the layer's lengths (replays
+ * advance them unseen by the host): every later host call that reads them
+ * (append, prefill, the other decodes, hwkv_seq_len, hwkv_row_len,
+ * hwkv_residency_bytes) first waits for the device (cudaDeviceSynchronize) and
+ * re-reads them; such calls cannot be captured. Arguments as hwkv_decode_step.
+ * During capture, make no other call on the cache from another thread.
+ */
+HWKV_API hwkv_status hwkv_decode_step_graph(hwkv_cache* cache, int32_t layer, const void* q,
+                                            const void* k_new, const void* v_new, float scale,
+                                            float* out, void* cuda_stream);
+
+/* Waits for cuda_stream, then copies the device lengths of every layer to the
+ * host copy (the calls above do this by themselves for graph-owned layers). */
+HWKV_API hwkv_status hwkv_sync_lens(hwkv_cache* cache, void* cuda_stream);
+
+/*
+ * Rows [row0, row0 + n_rows) of every layer restart empty (idle = 0: t_b = 0)
+ * or become idle (idle != 0: t_b = -1), e.g. when a request finishes and its
+ * batch slot is reused. Ring contents are left in place; the new length makes
+ * them unreachable. Stream-ordered (a cudaMemsetAsync per layer); may be captured.
+ */
+HWKV_API hwkv_status hwkv_reset_rows(hwkv_cache* cache, int32_t row0, int32_t n_rows,
+                                     int32_t idle, void* cuda_stream);
+
+/* Length t_b of one row (-1 = idle). */
+HWKV_API hwkv_status hwkv_row_len(const hwkv_cache* cache, int32_t layer, int32_t row, int64_t* t);
+
 /* Size of the device array hwkv_decode_attn_static keeps its scratch in. */
 #define HWKV_DECODE_STATIC_SCRATCH_BYTES (4u << 20)
 
@@ -171,18 +239,19 @@ HWKV_API hwkv_status hwkv_decode_step(hwkv_cache* cache, int32_t layer, const vo
  * (cudaMalloc and cudaFree can), and code issued during stream capture are
  * handed their inputs and outputs but cannot create scratch buffers.
  *
- * Same result and arguments as hwkv_decode_attn, but the per-tile partials
- * live in a fixed 4 MiB array inside this library's device image (present on
- * every GPU that loads the library until the process exits) instead of the
- * cache's workspace. It calls no cudaMalloc, cudaFree or allocating routine.
+ * Same result and arguments as hwkv_decode_attn, but the partial outputs and
+ * the work plan live in a fixed 4 MiB array inside this library's device image
+ * (present on every GPU that loads the library until the process exits)
+ * instead of the cache's workspace. It calls no cudaMalloc, cudaFree or allocating routine.
  * The first call on each device, with that device current, looks up the
  * array's device address (cudaGetSymbolAddress); make that first call before
  * any stream capture. The array keeps the last call's contents and nothing in
  * it needs to start at zero. All calls share it: calls whose kernels overlap
  * on the GPU (other streams, other caches) race and give wrong results.
- * Fails with HWKV_EINVAL when batch * n_kv_heads exceeds the tiles the array
- * holds ((4 MiB - 256) / (32 * head_dim + 64): 508 at head_dim 256, 1008
- * at 128, 1985 at 64), before anything is launched.
+ * It needs 2 * grid * (32 * head_dim + 64) bytes of partials (grid <= the SM
+ * count) plus 16 * (2 + batch * n_kv_heads) bytes of plan, both rounded up to
+ * 256: 2.5 MB + 16 B per ring on 152 SMs at head_dim 256. A layout that does
+ * not fit fails with HWKV_EINVAL before anything is launched.
  */
 HWKV_API hwkv_status hwkv_decode_attn_static(hwkv_cache* cache, int32_t layer, const void* q,
                                              float scale, float* out, void* cuda_stream);
@@ -272,15 +341,17 @@ HWKV_API hwkv_status hwkv_policy_load(const char* path, char* artifact, size_t a
 
 /*
  * Resident K+V bytes (Sec. 3.1, Eq. nominal-storage with C = t, bf16 K and V,
- * times batch): sum over KV heads of batch * min(cap, t) * head_dim * 2 * 2,
- * for one layer, or summed over all layers when layer == -1. Host-only.
+ * per row): sum over KV heads and rows b of min(cap, t_b) * head_dim * 2 * 2
+ * (idle rows hold nothing), for one layer, or summed over all layers when
+ * layer == -1. Host-only.
  */
 HWKV_API hwkv_status hwkv_residency_bytes(const hwkv_cache* cache, int32_t layer, uint64_t* bytes);
 
 /* Bytes of ring storage allocated (sum of batch * cap * head_dim * 4); layer -1 = all. */
 HWKV_API hwkv_status hwkv_allocated_ring_bytes(const hwkv_cache* cache, int32_t layer, uint64_t* bytes);
 
-/* Tokens held by `layer` so far (its t). */
+/* Tokens held by `layer` so far (its t) when every row holds the same number;
+ * HWKV_EINVAL when rows differ or are idle (use hwkv_row_len). */
 HWKV_API hwkv_status hwkv_seq_len(const hwkv_cache* cache, int32_t layer, int64_t* t);
 
 /* Ring capacity of (layer, kv_head): min(W, max_ctx), or max_ctx for full. */
@@ -297,8 +368,9 @@ HWKV_API hwkv_status hwkv_debug_copy_ring(const hwkv_cache* cache, int32_t layer
 
 /*
  * Synchronizes the device and reads the cache's kernel error word; returns
- * HWKV_EKERNEL (and clears the word) if a kernel gave up on a bounded wait or
- * saw an inconsistent index, else HWKV_OK.
+ * HWKV_EKERNEL (and clears the word) if a kernel gave up on a bounded wait,
+ * saw an inconsistent index, or a graph-mode step skipped a row at max_ctx,
+ * else HWKV_OK.
  */
 HWKV_API hwkv_status hwkv_sync_check(hwkv_cache* cache);
 

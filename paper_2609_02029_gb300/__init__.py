@@ -88,6 +88,13 @@ def lib():
             "hwkv_decode_attn": [_vp, _i32, _vp, ctypes.c_float, _vp, _vp],
             "hwkv_decode_attn_static": [_vp, _i32, _vp, ctypes.c_float, _vp, _vp],
             "hwkv_decode_step": [_vp, _i32, _vp, _vp, _vp, ctypes.c_float, _vp, _vp],
+            "hwkv_decode_step_graph": [_vp, _i32, _vp, _vp, _vp, ctypes.c_float, _vp, _vp],
+            "hwkv_append_rows": [_vp, _i32, _i32, _i32, _vp, _vp, _i64, _vp],
+            "hwkv_prefill_rows": [_vp, _i32, _i32, _i32, _vp, _vp, _vp, _i64, ctypes.c_float,
+                                  _vp, _vp],
+            "hwkv_sync_lens": [_vp, _vp],
+            "hwkv_reset_rows": [_vp, _i32, _i32, _i32, _vp],
+            "hwkv_row_len": [_vp, _i32, _i32, ctypes.POINTER(_i64)],
             "hwkv_residency_bytes": [_vp, _i32, _u64p],
             "hwkv_allocated_ring_bytes": [_vp, _i32, _u64p],
             "hwkv_seq_len": [_vp, _i32, ctypes.POINTER(_i64)],
@@ -187,6 +194,35 @@ def hwkv_decode_attn(cache, layer, q, scale, out, stream=None):
 def hwkv_decode_step(cache, layer, q, k_new, v_new, scale, out, stream=None):
     _check(lib().hwkv_decode_step(cache, layer, _ptr(q), _ptr(k_new), _ptr(v_new), scale,
                                   _ptr(out), _stream(stream)))
+
+
+def hwkv_decode_step_graph(cache, layer, q, k_new, v_new, scale, out, stream=None):
+    _check(lib().hwkv_decode_step_graph(cache, layer, _ptr(q), _ptr(k_new), _ptr(v_new), scale,
+                                        _ptr(out), _stream(stream)))
+
+
+def hwkv_append_rows(cache, layer, row0, n_rows, k, v, n, stream=None):
+    _check(lib().hwkv_append_rows(cache, layer, row0, n_rows, _ptr(k), _ptr(v), n,
+                                  _stream(stream)))
+
+
+def hwkv_prefill_rows(cache, layer, row0, n_rows, q, k, v, n, scale, out, stream=None):
+    _check(lib().hwkv_prefill_rows(cache, layer, row0, n_rows, _ptr(q), _ptr(k), _ptr(v), n,
+                                   scale, _ptr(out), _stream(stream)))
+
+
+def hwkv_sync_lens(cache, stream=None):
+    _check(lib().hwkv_sync_lens(cache, _stream(stream)))
+
+
+def hwkv_reset_rows(cache, row0, n_rows, idle=False, stream=None):
+    _check(lib().hwkv_reset_rows(cache, row0, n_rows, 1 if idle else 0, _stream(stream)))
+
+
+def hwkv_row_len(cache, layer, row):
+    v = ctypes.c_int64(0)
+    _check(lib().hwkv_row_len(cache, layer, row, ctypes.byref(v)))
+    return v.value
 
 
 def hwkv_decode_attn_static(cache, layer, q, scale, out, stream=None):

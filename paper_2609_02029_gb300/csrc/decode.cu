@@ -4,12 +4,14 @@
 // each GQA query-head group reads its KV head's own slice).
 //
 // Work decomposition. For one layer, every (batch row b, KV head h) ring holds
-// n_h = min(t, cap_h) resident slots; after the append of token t-1 these are
-// exactly the positions J_{t-1}(W_h), so the softmax runs over all of them and
-// slot order does not matter. Rings are cut into tiles of equal length
-// (tile_len tokens, a multiple of 64), so a full-history head gets many tiles
-// and a short-window head few: the split count follows the resident length and
-// all window levels share one launch. A persistent grid walks the tile list.
+// n = min(t_b, cap_h) resident slots; after the append of token t_b - 1 these
+// are exactly the positions J_{t_b - 1}(W_h), so the softmax runs over all of
+// them and slot order does not matter. The rings are laid end to end and every
+// CTA of the persistent grid takes an equal share of their tokens, cut at ring
+// boundaries into segments (the plan is made on the GPU from the per-row
+// lengths, see make_device_plan): a full-history ring is split over many CTAs,
+// short-window rings are read whole by one, and all window levels share one
+// launch.
 //
 // Inside a CTA: warp 4 is the producer -- one lane issues 2-D TMA loads of
 // 64-token stages of K and V (128-byte swizzle, one box per 64 channels) into
@@ -22,6 +24,8 @@
 // heads of a GQA group share every K/V byte read. Each warp leaves a partial
 // (max, sum, unnormalised output); the four warps merge theirs in shared memory
 // into one partial per tile, and the combine kernel merges the tiles of a head.
+#include <mutex>
+
 #include "hwkv_internal.cuh"
 
 namespace hwkv {
@@ -33,34 +37,236 @@ struct TileInfo {
   int64_t start;  // first slot of the tile
   int len;        // slots in the tile (>= 1)
   int64_t k_row, v_row;
+  int tile;       // partial slot of the tile
+  int64_t s_new;  // fused step: ring slot that receives the new token
+  bool single;    // the tile covers the whole ring: its output is final
 };
 
-__device__ __forceinline__ TileInfo locate_tile(const DecodeParams& p, int tile) {
-  TileInfo ti;
-  if (p.tiles != nullptr) {  // explicit tile table
+// ---- device-side plan (per-row lengths read on the GPU)
+//
+// Ring u (unit order u = b * n_units + h) holds n_u = min(len_b + lens_inc,
+// cap_h) keys (0 for an idle row or a row whose step would pass max_ctx), read in
+// q_u = ceil(n_u / 64) stages (a partial last stage is loaded whole). A segment
+// (a piece of one ring read by one CTA) also has a fixed cost of F stages (the
+// query load, the cross-warp merge and the partial write). The rings are laid
+// end to end on a cost line in stage units, ring u taking F + q_u from L_u =
+// sum_{v<u} w_v (w_v = q_v + F for a ring with keys, 0 otherwise), total Lt. CTA
+// c takes the line [floor(c Lt / G'), floor((c + 1) Lt / G')), G' = min(gridDim.x,
+// Lt), and reads the stages it covers (a point in a ring's F-stretch maps to the
+// ring's first stage). So every CTA gets the same cost to one stage, a CTA that
+// starts more rings reads fewer keys, cuts fall on stage boundaries (neighbouring
+// CTAs never load the same stage), and no CTA below G' is empty. Only a CTA's
+// first and last segment can belong to a ring other CTAs also read; every other
+// segment is a whole ring and gives that ring's output at once. A partial needs
+// two slots per CTA: 2c for the first segment, 2c + 1 for the last.
+//
+// Every warp derives the plan in registers (no block barrier): the rings are
+// spread over the lanes (u = 32 r + lane), the first 256 kept in registers and
+// further ones re-read. Warp 0 of CTA 0 also stores Lt, G', F and every ring's
+// (L_u, n_u) for the combine kernel.
+constexpr int kPlanRegs = 8;
+
+struct DevPlan {
+  int64_t count;  // keys of this CTA (0: idle)
+  int64_t off0;   // first slot of the first segment, within ring u0
+  int u0;
+};
+
+__device__ __forceinline__ int dev_unit_len(const DecodeParams& p, int u, int32_t& len_b) {
+  const int b = u / p.n_units;
+  const int h = u - b * p.n_units;
+  len_b = p.lens[b];
+  if (len_b < 0 || (int64_t)len_b + p.lens_inc > p.max_ctx) return 0;
+  const int64_t n = (int64_t)len_b + p.lens_inc;
+  return (int)(n < p.u[h].cap ? n : p.u[h].cap);
+}
+
+__device__ __forceinline__ long long warp_incl_scan(long long v, int lane) {
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const long long x = __shfl_up_sync(0xffffffffu, v, off);
+    if (lane >= off) v += x;
+  }
+  return v;
+}
+
+// called by whole warps; every lane returns the same plan
+__device__ __forceinline__ long long stages_of(long long n) {
+  return (n + kStageTokens - 1) / kStageTokens;
+}
+
+__device__ DevPlan make_device_plan(const DecodeParams& p, bool write_table) {
+  const int lane = threadIdx.x & 31;
+  const int U = p.batch * p.n_units;
+  const int R = (U + 31) / 32;
+  const long long F = p.seg_cost;  // stages
+  int nreg[kPlanRegs];
+  long long Lt = 0, N = 0;
+#pragma unroll
+  for (int r = 0; r < kPlanRegs; ++r) {
+    const int u = r * 32 + lane;
+    int n = 0;
+    if (r < R && u < U) {
+      int32_t L;
+      n = dev_unit_len(p, u, L);
+      if (write_table && u % p.n_units == 0 && L >= 0 && (int64_t)L + p.lens_inc > p.max_ctx)
+        atomicOr(p.err, kErrCapacity);
+    }
+    nreg[r] = n;
+    Lt += n > 0 ? stages_of(n) + F : 0;
+    N += n;
+  }
+  for (int r = kPlanRegs; r < R; ++r) {  // rings beyond the register cache
+    const int u = r * 32 + lane;
+    if (u < U) {
+      int32_t L;
+      const int n = dev_unit_len(p, u, L);
+      Lt += n > 0 ? stages_of(n) + F : 0;
+      N += n;
+      if (write_table && u % p.n_units == 0 && L >= 0 && (int64_t)L + p.lens_inc > p.max_ctx)
+        atomicOr(p.err, kErrCapacity);
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    Lt += __shfl_xor_sync(0xffffffffu, Lt, off);
+    N += __shfl_xor_sync(0xffffffffu, N, off);
+  }
+
+  const long long G = min((long long)gridDim.x, max(Lt, 1LL));
+  const bool mine = (long long)blockIdx.x < G && Lt > 0;
+  const long long A0 = mine ? (long long)blockIdx.x * Lt / G : 0;
+  const long long A1 = mine ? ((long long)blockIdx.x + 1) * Lt / G : 0;
+  // line point -> key: the ring whose stretch [L_u, L_u + F + q_u) holds the point
+  long long a = -1, b = mine && A1 >= Lt ? N : -1;  // A1 = Lt: up to the last key
+  long long sa = 0;
+  int ua = 0;
+  long long carry_w = 0, carry_n = 0;
+  for (int r = 0; r < R && ((mine && (a < 0 || b == -1)) || write_table); ++r) {
+    int n = 0;
+#pragma unroll
+    for (int i = 0; i < kPlanRegs; ++i)
+      if (i == r) n = nreg[i];
+    const int u = r * 32 + lane;
+    if (r >= kPlanRegs && u < U) {
+      int32_t L;
+      n = dev_unit_len(p, u, L);
+    }
+    const long long w = n > 0 ? stages_of(n) + F : 0;
+    const long long iw = warp_incl_scan(w, lane), in = warp_incl_scan(n, lane);
+    const long long Lu = carry_w + iw - w, su = carry_n + in - n;
+    if (write_table && u < U) {
+      p.plan[4 + 2 * u] = Lu;
+      p.plan[5 + 2 * u] = n;
+    }
+    if (mine && a < 0) {
+      const unsigned hit = __ballot_sync(0xffffffffu, w > 0 && Lu <= A0 && A0 < Lu + w);
+      if (hit) {
+        const int src = __ffs(hit) - 1;
+        const long long lu = __shfl_sync(0xffffffffu, Lu, src);
+        const long long s0 = __shfl_sync(0xffffffffu, su, src);
+        a = s0 + max(0LL, A0 - lu - F) * kStageTokens;
+        sa = s0;
+        ua = r * 32 + src;
+      }
+    }
+    if (mine && b == -1) {
+      const unsigned hit = __ballot_sync(0xffffffffu, w > 0 && Lu <= A1 && A1 < Lu + w);
+      if (hit) {
+        const int src = __ffs(hit) - 1;
+        const long long lu = __shfl_sync(0xffffffffu, Lu, src);
+        const long long s1 = __shfl_sync(0xffffffffu, su, src);
+        b = s1 + max(0LL, A1 - lu - F) * kStageTokens;
+      }
+    }
+    carry_w += __shfl_sync(0xffffffffu, iw, 31);
+    carry_n += __shfl_sync(0xffffffffu, in, 31);
+  }
+  DevPlan dp;
+  dp.count = mine && a >= 0 && b > a ? b - a : 0;
+  dp.u0 = ua;
+  dp.off0 = a - sa;  // key a lies in ring ua
+  if (write_table && lane == 0) {
+    p.plan[0] = Lt;
+    p.plan[1] = G;
+    p.plan[2] = F;
+  }
+  return dp;
+}
+
+// The tiles of one CTA, in order. Ring mode: the CTA's segments (above). Table
+// mode: tiles blockIdx.x, + gridDim.x, ... of the explicit tile list.
+struct TileWalker {
+  int j = 0, count = 0;  // table mode
+  // ring mode cursor
+  int64_t rem = 0, start = 0;
+  int u = 0, n = 0;
+  int32_t len_b = 0;
+  bool first = true, advance = false;
+
+  __device__ void init(const DecodeParams& p, const DevPlan& dp) {
+    if (p.tiles != nullptr) {
+      count = blockIdx.x < p.n_tiles ? (p.n_tiles - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+      return;
+    }
+    rem = dp.count;
+    if (rem > 0) {
+      u = dp.u0;
+      start = dp.off0;
+      n = dev_unit_len(p, u, len_b);
+    }
+  }
+
+  __device__ bool next(const DecodeParams& p, TileInfo& ti) {
+    if (p.tiles != nullptr) {
+      if (j >= count) return false;
+      table_tile(p, blockIdx.x + j * gridDim.x, ti);
+      ++j;
+      return true;
+    }
+    if (rem <= 0) return false;
+    if (advance) {  // the next ring that holds anything
+      const int U = p.batch * p.n_units;
+      do {
+        if (++u >= U) {  // the plan promised more tokens: lengths changed under the kernel
+          atomicOr(p.err, kErrBadIndex);
+          rem = 0;
+          return false;
+        }
+        n = dev_unit_len(p, u, len_b);
+      } while (n == 0);
+      start = 0;
+    }
+    ti.b = u / p.n_units;
+    ti.h = u - ti.b * p.n_units;
+    const DecodeUnit& du = p.u[ti.h];
+    const int64_t len = min((int64_t)n - start, rem);
+    ti.start = start;
+    ti.len = (int)len;
+    ti.k_row = du.k_row0 + (int64_t)ti.b * du.cap + start;
+    ti.v_row = du.v_row0 + (int64_t)ti.b * du.cap + start;
+    ti.s_new = (int64_t)len_b % du.cap;
+    ti.single = start == 0 && len == n;
+    ti.tile = 2 * (int)blockIdx.x + (first ? 0 : 1);
+    rem -= len;
+    first = false;
+    advance = true;
+    return true;
+  }
+
+  __device__ static void table_tile(const DecodeParams& p, int tile, TileInfo& ti) {
     const CalibTile ct = p.tiles[tile];
+    ti.tile = tile;
     ti.b = ct.q_row;
     ti.h = ct.h;
     ti.start = 0;
     ti.len = ct.len;
     ti.k_row = ct.k_row;
     ti.v_row = ct.v_row;
-    return ti;
+    ti.s_new = -1;
+    ti.single = false;
   }
-  ti.b = tile / p.tiles_per_b;
-  const int lt = tile - ti.b * p.tiles_per_b;
-  int h = 0;
-  while (h + 1 < p.n_units && lt >= p.u[h].tile_begin + p.u[h].n_tiles) ++h;
-  ti.h = h;
-  const DecodeUnit& u = p.u[h];
-  const int i = lt - u.tile_begin;
-  ti.start = (int64_t)i * p.tile_len;
-  const int64_t rem = (int64_t)u.n_valid - ti.start;
-  ti.len = (int)(rem < p.tile_len ? rem : p.tile_len);
-  ti.k_row = u.k_row0 + (int64_t)ti.b * u.cap + ti.start;
-  ti.v_row = u.v_row0 + (int64_t)ti.b * u.cap + ti.start;
-  return ti;
-}
+};
 
 // named barrier of the four consumer warps (the producer warp does not take part)
 __device__ __forceinline__ void consumer_sync() {
@@ -110,8 +316,11 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     fence_barrier_init();
   }
   __syncthreads();
-  grid_dep_wait();    // the ring append and q come from kernels launched before
+  grid_dep_wait();    // the ring append, q and the lengths come from kernels launched before
   grid_dep_launch();  // the combine kernel may start launching
+  DevPlan dplan{};
+  if (p.tiles == nullptr)  // each warp plans for itself; warp 0 of CTA 0 leaves the table
+    dplan = make_device_plan(p, blockIdx.x == 0 && warp == 0);
 
   if (warp == kDecodeWarps) {
     // ------------------------------------------------------------ producer
@@ -120,8 +329,10 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     prefetch_tensormap(&v_map);
     uint32_t it = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; ok && tile < p.n_tiles; tile += gridDim.x) {
-      const TileInfo ti = locate_tile(p, tile);
+    TileWalker wk;
+    wk.init(p, dplan);
+    TileInfo ti;
+    while (ok && wk.next(p, ti)) {
       const int n_st = (ti.len + kStageTokens - 1) / kStageTokens;
       for (int st = 0; st < n_st; ++st, ++it) {
         const int s = it % STAGES;
@@ -163,8 +374,10 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
   // reaches the same named barriers.
   bool aborted = false;
 
-  for (int tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x) {
-    const TileInfo ti = locate_tile(p, tile);
+  TileWalker wk;
+  wk.init(p, dplan);
+  TileInfo ti;
+  while (wk.next(p, ti)) {
     const int n_st = (ti.len + kStageTokens - 1) / kStageTokens;
 
     // Q^T as mma B fragments: b0 = channels 16kk + qk + {0,1}, b1 = +8; column = head qn
@@ -199,13 +412,13 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
       if (p.k_new != nullptr) {
         // fused step: the new token's slot may lie in this stage; the warp owning that
         // row replaces the staged (stale) row with the new K/V and writes the ring row
-        const int64_t row_in = (int64_t)p.u[ti.h].s_new - (ti.start + (int64_t)st * kStageTokens);
+        const int64_t row_in = ti.s_new - (ti.start + (int64_t)st * kStageTokens);
         if (row_in >= w * 16 && row_in < w * 16 + 16) {
           const int r = (int)row_in;
           const __nv_bfloat16* src_k = p.k_new + ((int64_t)ti.b * p.n_units + ti.h) * D;
           const __nv_bfloat16* src_v = p.v_new + ((int64_t)ti.b * p.n_units + ti.h) * D;
-          const int64_t ring_row = ti.k_row - ti.start + p.u[ti.h].s_new;  // K region row
-          const int64_t vring_row = ti.v_row - ti.start + p.u[ti.h].s_new;
+          const int64_t ring_row = ti.k_row - ti.start + ti.s_new;  // K region row
+          const int64_t vring_row = ti.v_row - ti.start + ti.s_new;
           for (int idx = lane; idx < 2 * (D / 8); idx += 32) {
             const int isv = idx >= D / 8;
             const int ch = isv ? idx - D / 8 : idx;  // 16-byte chunk of the row
@@ -314,8 +527,8 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     {
       // one tile covers the whole ring: this is the final output, normalised here;
       // otherwise leave the tile's partial for the combine kernel
-      const bool single = p.tiles == nullptr && p.u[ti.h].n_tiles == 1;
-      float* po = p.part_o + (int64_t)tile * kMaxGroup * D;
+      const bool single = ti.single;
+      float* po = p.part_o + (int64_t)ti.tile * kMaxGroup * D;
       float* fo = p.out + ((int64_t)ti.b * p.n_q_heads + (int64_t)ti.h * p.group) * D;
       for (int n = 0; n < p.group; ++n) {
         float M = -INFINITY;
@@ -338,18 +551,18 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
           dst[i] = acc * scale_out;
         }
         if (!single && w == 0 && lane == 0)
-          p.part_ml[(int64_t)tile * kMaxGroup + n] = make_float2(M, L);
+          p.part_ml[(int64_t)ti.tile * kMaxGroup + n] = make_float2(M, L);
       }
     }
   }
 }
 
-// Log-sum-exp merge of the tile partials of one (batch row, query head):
+// Log-sum-exp merge of the segment partials of one (batch row, query head):
 // o = sum_j 2^{(m_j - M) c} o_j / sum_j 2^{(m_j - M) c} l_j, M = max_j m_j.
-// One CTA of 8 warps per (batch row, query head): warp w sums tiles w, w+8, ...
+// One CTA of 8 warps per (batch row, query head): warp w sums partials w, w+8, ...
 // over all channels (each lane D/32 consecutive channels, vector loads); the
 // eight partial sums are added in shared memory in warp order (deterministic).
-// Heads whose ring is a single tile were written by the split kernel.
+// Rings read whole by one CTA were written by the split kernel.
 constexpr int kCombineWarps = 8;
 
 template <int D>
@@ -364,16 +577,35 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
   const int qh = bq - b * p.n_q_heads;
   const int h = qh / p.group;
   const int n = qh - h * p.group;
-  const DecodeUnit& u = p.u[h];
-  const int n_t = u.n_tiles;
-  if (n_t <= 1) return;
-  const int64_t tile0 = (int64_t)b * p.tiles_per_b + u.tile_begin;
+  // the ring's segments: its stages span the cost line [L + F, L + F + q), read
+  // by CTAs c1 .. c2 of the split launch; the first segment's partial sits in
+  // slot 2 c1 (the ring starts that CTA's range) or 2 c1 + 1 (it is that CTA's
+  // last segment), every later one in slot 2 c (the ring starts that CTA's range)
+  const int u = b * p.n_units + h;
+  const long long Lt = p.plan[0], G = p.plan[1], F = p.plan[2];
+  const long long Lu = p.plan[4 + 2 * u], nu = p.plan[5 + 2 * u];
+  // every ring of an active row holds >= 1 key; the split kernel has finished
+  // reading the lengths, so the row can advance now
+  if (p.lens_inc && qh == 0 && threadIdx.x == 0 && p.plan[5 + 2 * (b * p.n_units)] > 0)
+    p.lens[b] += 1;
+  if (nu == 0) {  // idle row (or a row at max_ctx): zero output
+    for (int i = threadIdx.x; i < D; i += blockDim.x)
+      p.out[((int64_t)b * p.n_q_heads + qh) * D + i] = 0.f;
+    return;
+  }
+  const long long qu = (nu + kStageTokens - 1) / kStageTokens;
+  const long long c1 = ((Lu + F + 1) * G - 1) / Lt;   // the CTA with the first stage
+  const long long c2 = ((Lu + F + qu) * G - 1) / Lt;  // the CTA with the last stage
+  if (c1 == c2) return;  // one CTA read the whole ring and wrote the output
+  const int n_t = (int)(c2 - c1 + 1);
+  const int64_t slot0 = 2 * c1 + (c1 * Lt / G >= Lu ? 0 : 1);
+  auto slot = [&](int j) -> int64_t { return j == 0 ? slot0 : 2 * (c1 + j); };
   const float c = p.scale_log2;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   float mx = -INFINITY;
   for (int j = threadIdx.x; j < n_t; j += blockDim.x)
-    mx = fmaxf(mx, p.part_ml[(tile0 + j) * kMaxGroup + n].x);
+    mx = fmaxf(mx, p.part_ml[slot(j) * kMaxGroup + n].x);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   if (lane == 0) s_max[w] = mx;
@@ -387,10 +619,10 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
   for (int e = 0; e < PER; ++e) acc[e] = 0.f;
   float den = 0.f;
   for (int j = w; j < n_t; j += kCombineWarps) {
-    const float2 ml = p.part_ml[(tile0 + j) * kMaxGroup + n];
+    const float2 ml = p.part_ml[slot(j) * kMaxGroup + n];
     const float wgt = ml.x == -INFINITY ? 0.f : ex2((ml.x - M) * c);
     den += wgt * ml.y;
-    const float* src = p.part_o + ((tile0 + j) * kMaxGroup + n) * D + lane * PER;
+    const float* src = p.part_o + (slot(j) * kMaxGroup + n) * D + lane * PER;
 #pragma unroll
     for (int e = 0; e < PER; e += 2) {
       const float2 v = *reinterpret_cast<const float2*>(src + e);
@@ -422,15 +654,37 @@ int decode_smem_bytes(int head_dim) {
   }
 }
 
+// The shared-memory opt-in of the split kernels, once per device (host calls
+// made before any stream capture, e.g. hwkv_alloc, take care of it).
+cudaError_t decode_prepare_device() {
+  constexpr int kMaxDevices = 64;
+  static std::mutex mu;
+  static bool done[kMaxDevices] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (done[dev]) return cudaSuccess;
+  e = cudaFuncSetAttribute(decode_split_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           DecodeCfg<64>::kSmem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(decode_split_kernel<128>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeCfg<128>::kSmem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(decode_split_kernel<256>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeCfg<256>::kSmem);
+  if (e == cudaSuccess) done[dev] = true;
+  return e;
+}
+
 template <int D>
 static cudaError_t launch_decode_t(const DecodeParams& p, const CUtensorMap& kmap,
                                    const CUtensorMap& vmap, int grid, cudaStream_t s) {
-  const int smem = DecodeCfg<D>::kSmem;
-  cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = decode_prepare_device();
   if (e != cudaSuccess) return e;
-  return launch_pdl(decode_split_kernel<D>, dim3(grid), dim3((kDecodeWarps + 1) * 32), smem, s,
-                    kmap, vmap, p);
+  return launch_pdl(decode_split_kernel<D>, dim3(grid), dim3((kDecodeWarps + 1) * 32),
+                    DecodeCfg<D>::kSmem, s, kmap, vmap, p);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& kmap, const CUtensorMap& vmap,
@@ -551,9 +805,6 @@ cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cuda
 }
 
 cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s) {
-  bool any = false;  // nothing to merge when every ring is a single tile
-  for (int h = 0; h < p.n_units; ++h) any |= p.u[h].n_tiles > 1;
-  if (!any) return cudaSuccess;
   const dim3 grid(p.batch * p.n_q_heads), block(kCombineWarps * 32);
   switch (head_dim) {
     case 64: return launch_pdl(decode_combine_kernel<64>, grid, block, 0, s, p);

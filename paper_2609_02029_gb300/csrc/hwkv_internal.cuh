@@ -18,22 +18,21 @@ constexpr int kMaxKvHeads = 64;
 constexpr int kMaxGroup = 8;          // query heads per KV head handled by one mma n-tile
 constexpr int kDecodeWarps = 4;       // consumer warps per decode CTA
 constexpr int kStageTokens = 64;      // tokens per pipeline stage (16 per consumer warp)
-constexpr int kCombineMaxTiles = 4096;  // tiles of one ring the combine kernel can merge
 constexpr int kSlabBytes = 64 * 128;  // one TMA box: 64 rows x 128 B (64 bf16)
 
 // error word bits (set with atomicOr, read by hwkv_sync_check)
 constexpr int kErrWaitTimeout = 1;
 constexpr int kErrBadIndex = 2;
+constexpr int kErrCapacity = 4;  // a device-length step found a row at max_ctx (row skipped)
+
+constexpr int kMaxBatch = 256;
+constexpr int kDecodeSlots = 512;  // decode partial slots in the cache workspace (2 per CTA)
 
 // ------------------------------------------------------------------ decode
 struct DecodeUnit {
   int64_t k_row0;   // arena row of (this KV head, batch row 0) in the K region
   int64_t v_row0;   // same in the V region
   int64_t cap;      // ring capacity; batch row b starts at row0 + b * cap
-  int32_t n_valid;  // resident slots: min(t, cap)
-  int32_t n_tiles;  // tiles this head's ring is split into, per batch row
-  int32_t tile_begin;  // first tile of this head within one batch row's tile list
-  int32_t s_new;       // fused step: ring slot that receives the new token
 };
 
 // a tile of explicit key rows (SeqCalib replay): rows k_row.. / v_row.. of the trace
@@ -43,18 +42,18 @@ struct CalibTile {
   int32_t len, q_row, h, pad;
 };
 
+// Ring mode (tiles == nullptr): the rings of one layer, planned on the GPU from the
+// per-row lengths. Table mode: an explicit tile list (SeqCalib replay).
 struct DecodeParams {
   int32_t n_units;      // KV heads of the layer
   int32_t batch;
   int32_t group;        // G = n_q_heads / n_kv_heads
   int32_t n_q_heads;
-  int32_t tile_len;     // tokens per tile, multiple of kStageTokens
-  int32_t tiles_per_b;  // sum of n_tiles over heads
-  int32_t n_tiles;      // batch * tiles_per_b
+  int32_t n_tiles;      // table mode: tiles in `tiles`
   float scale_log2;     // scale * log2(e)
   const __nv_bfloat16* q;  // [batch][n_q_heads][D]
-  float* part_o;           // [n_tiles][kMaxGroup][D]: unnormalised tile outputs
-  float2* part_ml;         // [n_tiles][kMaxGroup]: (max logit, sum of weights)
+  float* part_o;           // [slots][kMaxGroup][D]: unnormalised partial outputs
+  float2* part_ml;         // [slots][kMaxGroup]: (max logit, sum of weights)
   float* out;              // [batch][n_q_heads][D]
   int* err;
   // fused step (append the new token, then attend): k_new/v_new [batch][n_units][D];
@@ -62,9 +61,15 @@ struct DecodeParams {
   const __nv_bfloat16* k_new;  // null: plain decode over the current ring contents
   const __nv_bfloat16* v_new;
   __nv_bfloat16* arena;        // K/V rows: row r at arena + r * D
-  // table mode (SeqCalib replay): tiles[n_tiles] replace the ring plan; every tile
-  // leaves a partial (no single-tile shortcut)
-  const CalibTile* tiles;
+  const CalibTile* tiles;      // table mode: tiles[n_tiles]; every tile leaves a partial
+  // ring mode: per-row lengths of this layer on the device, [batch]: tokens held by
+  // row b before this call, -1 = idle row. With lens_inc = 1 (fused step) the new
+  // token counts and the combine kernel advances every active row by one.
+  int32_t* lens;
+  int32_t lens_inc;
+  int64_t max_ctx;      // rows whose step would pass max_ctx are skipped (kErrCapacity)
+  int32_t seg_cost;     // fixed cost of a segment, in 64-key stages (F of the plan)
+  int64_t* plan;        // [4 + 2 * batch * n_units]: Lt, G, F, -, then (L_u, n_u) per ring
   DecodeUnit u[kMaxKvHeads];
 };
 
@@ -85,8 +90,10 @@ struct AppendUnit {
 };
 
 struct AppendParams {
-  int32_t n_units, batch;
-  int64_t t0;      // position of the first new token
+  int32_t n_units, batch;  // batch = rows of this call, cache rows row0 .. row0 + batch - 1
+  int32_t row0;
+  int32_t* lens;   // the layer's per-row lengths on the device; row r gets t0[r - row0] + n
+  int32_t t0[kMaxBatch];  // position of the first new token, per row of the call
   int64_t n;       // new tokens
   int64_t d;       // head_dim
   const __nv_bfloat16* k;  // [batch][n][n_units][d]
@@ -103,7 +110,8 @@ struct PrefillUnit {
 };
 
 struct PrefillParams {
-  int32_t n_units, batch, group, n_q_heads;
+  int32_t n_units, batch, group, n_q_heads;  // batch = rows of this call
+  int32_t row0;                              // first cache row of the call
   int64_t t0;  // first chunk position (tokens already in the cache)
   int64_t n;   // chunk length
   float scale_log2;
@@ -127,6 +135,7 @@ cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtens
                               const CUtensorMap& ck_map, const CUtensorMap& cv_map,
                               const CUtensorMap& ring_map, cudaStream_t s);
 int decode_smem_bytes(int head_dim);
+cudaError_t decode_prepare_device();  // one-time kernel attributes on the current device
 
 // ------------------------------------------------------------ device PTX
 #if defined(__CUDACC__)

@@ -56,8 +56,8 @@ struct Layout {
   std::vector<Unit> units;  // [layer * n_kv_heads + h]
   int64_t rows = 0;         // K rows (= V rows)
   size_t ring_bytes = 0;    // K + V
-  size_t part_o_off = 0, part_ml_off = 0, err_off = 0, total = 0;
-  int max_tiles = 0;
+  size_t part_o_off = 0, part_ml_off = 0, err_off = 0, lens_off = 0, plan_off = 0, total = 0;
+  int slots = 0;  // decode partial slots: two per CTA of a split launch
 };
 
 hwkv_status validate(const hwkv_policy* p) {
@@ -107,12 +107,16 @@ Layout make_layout(const hwkv_policy* p) {
   for (auto& u : L.units) u.v_row0 = u.k_row0 + L.rows;
   const size_t row_bytes = (size_t)p->head_dim * 2;
   L.ring_bytes = (size_t)(2 * L.rows) * row_bytes;
-  L.max_tiles = std::max(2048, 2 * p->batch * p->n_kv_heads);
+  L.slots = kDecodeSlots;
   L.part_o_off = align_up(L.ring_bytes, kAlign);
-  L.part_ml_off =
-      align_up(L.part_o_off + (size_t)L.max_tiles * kMaxGroup * p->head_dim * 4, kAlign);
-  L.err_off = align_up(L.part_ml_off + (size_t)L.max_tiles * kMaxGroup * 8, kAlign);
-  L.total = align_up(L.err_off + 64, kAlign);
+  L.part_ml_off = align_up(L.part_o_off + (size_t)L.slots * kMaxGroup * p->head_dim * 4, kAlign);
+  L.err_off = align_up(L.part_ml_off + (size_t)L.slots * kMaxGroup * 8, kAlign);
+  // per-row lengths on the device, [layer][batch] int32, then the decode plan
+  // table (int64): the cost line's length, the CTAs, the segment cost, and per
+  // ring its place on the line and its keys
+  L.lens_off = align_up(L.err_off + 64, kAlign);
+  L.plan_off = align_up(L.lens_off + (size_t)p->n_layers * p->batch * 4, kAlign);
+  L.total = align_up(L.plan_off + (size_t)(4 + 2 * p->batch * p->n_kv_heads) * 8, kAlign);
   return L;
 }
 
@@ -137,7 +141,12 @@ struct hwkv_cache {
   hwkv_policy pol;
   std::vector<int64_t> windows;
   Layout lay;
-  std::vector<int64_t> t;  // tokens held, per layer
+  // tokens held per (layer, row), -1 = idle row: the host copy of the device
+  // length array. A layer that has had a graph-mode step is advanced on the
+  // device without the host knowing (graph replays), so its copy is re-read
+  // before every use (dev_owned).
+  mutable std::vector<int64_t> t;
+  std::vector<char> dev_owned;  // per layer
   uint8_t* arena = nullptr;
   bool owns_arena = false;
   int num_sms = 0;
@@ -147,6 +156,21 @@ struct hwkv_cache {
   float* part_o() const { return reinterpret_cast<float*>(arena + lay.part_o_off); }
   float2* part_ml() const { return reinterpret_cast<float2*>(arena + lay.part_ml_off); }
   int* err() const { return reinterpret_cast<int*>(arena + lay.err_off); }
+  int32_t* lens(int layer) const {
+    return reinterpret_cast<int32_t*>(arena + lay.lens_off) + (size_t)layer * pol.batch;
+  }
+  int64_t* plan() const { return reinterpret_cast<int64_t*>(arena + lay.plan_off); }
+  int64_t& row_t(int layer, int b) { return t[(size_t)layer * pol.batch + b]; }
+  int64_t row_t(int layer, int b) const { return t[(size_t)layer * pol.batch + b]; }
+  // true (and the length) when every row of the layer holds the same number of tokens
+  bool uniform(int layer, int64_t* len) const {
+    const int64_t t0 = row_t(layer, 0);
+    for (int b = 1; b < pol.batch; ++b)
+      if (row_t(layer, b) != t0) return false;
+    if (t0 < 0) return false;
+    *len = t0;
+    return true;
+  }
 };
 
 extern "C" {
@@ -177,13 +201,23 @@ hwkv_status hwkv_alloc(const hwkv_policy* policy, void* dev_arena, size_t arena_
     return fail(HWKV_EINVAL, "dev_arena must be %zu-byte aligned", kAlign);
   auto encode = get_encode();
   if (!encode) return fail(HWKV_ECUDA, "cuTensorMapEncodeTiled entry point unavailable");
+  {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return fail(HWKV_ECUDA, "device query failed");
+    if (2 * sms > kDecodeSlots)
+      return fail(HWKV_EUNSUPPORTED, "%d SMs need more than the %d decode partial slots", sms,
+                  kDecodeSlots);
+  }
 
   hwkv_cache* c = new hwkv_cache();
   c->pol = *policy;
   c->windows.assign(policy->windows, policy->windows + (size_t)policy->n_layers * policy->n_kv_heads);
   c->pol.windows = c->windows.data();
   c->lay = std::move(lay);
-  c->t.assign(policy->n_layers, 0);
+  c->t.assign((size_t)policy->n_layers * policy->batch, 0);
+  c->dev_owned.assign(policy->n_layers, 0);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -201,6 +235,12 @@ hwkv_status hwkv_alloc(const hwkv_policy* policy, void* dev_arena, size_t arena_
       return fail(HWKV_ENOMEM, "cudaMalloc(%zu) failed: %s", c->lay.total, cudaGetErrorString(e));
     }
     c->owns_arena = true;
+  }
+  e = decode_prepare_device();
+  if (e != cudaSuccess) {
+    if (c->owns_arena) cudaFree(c->arena);
+    delete c;
+    return fail(HWKV_ECUDA, "decode kernel attributes: %s", cudaGetErrorString(e));
   }
   e = cudaMemsetAsync(c->arena, 0, c->lay.total, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
@@ -240,12 +280,40 @@ static hwkv_status check_layer(const hwkv_cache* c, int32_t layer) {
   return HWKV_OK;
 }
 
-static AppendParams append_params(const hwkv_cache* c, int32_t layer, const void* k,
-                                  const void* v, int64_t n) {
+// Host calls that read the host copy of a layer's lengths: if graph-mode steps
+// own the layer, wait for the device and re-read its lengths first.
+static hwkv_status refresh_lens(const hwkv_cache* c, int32_t layer) {
+  if (!c->dev_owned[layer]) return HWKV_OK;
+  std::vector<int32_t> host(c->pol.batch);
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess)
+    e = cudaMemcpy(host.data(), c->lens(layer), host.size() * 4, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "length copy: %s", cudaGetErrorString(e));
+  for (int b = 0; b < c->pol.batch; ++b) c->t[(size_t)layer * c->pol.batch + b] = host[b] < 0 ? -1 : host[b];
+  return HWKV_OK;
+}
+
+static hwkv_status check_fresh(const hwkv_cache* c, int32_t layer) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  return refresh_lens(c, layer);
+}
+
+static hwkv_status check_rows(const hwkv_cache* c, int32_t row0, int32_t n_rows) {
+  if (row0 < 0 || n_rows <= 0 || (int64_t)row0 + n_rows > c->pol.batch)
+    return fail(HWKV_EINVAL, "rows [%d, %d + %d) outside the batch of %d", row0, row0, n_rows,
+                c->pol.batch);
+  return HWKV_OK;
+}
+
+static AppendParams append_params(const hwkv_cache* c, int32_t layer, int32_t row0,
+                                  int32_t n_rows, const void* k, const void* v, int64_t n) {
   AppendParams p{};
   p.n_units = c->pol.n_kv_heads;
-  p.batch = c->pol.batch;
-  p.t0 = c->t[layer];
+  p.batch = n_rows;
+  p.row0 = row0;
+  p.lens = c->lens(layer);
+  for (int b = 0; b < n_rows; ++b) p.t0[b] = (int32_t)c->row_t(layer, row0 + b);
   p.n = n;
   p.d = c->pol.head_dim;
   p.k = static_cast<const __nv_bfloat16*>(k);
@@ -259,42 +327,66 @@ static AppendParams append_params(const hwkv_cache* c, int32_t layer, const void
   return p;
 }
 
-hwkv_status hwkv_append(hwkv_cache* c, int32_t layer, const void* k, const void* v, int64_t n,
-                        void* cuda_stream) {
-  hwkv_status st = check_layer(c, layer);
+// rows [row0, row0 + n_rows) may each append n tokens: active, and within max_ctx
+static hwkv_status check_room(const hwkv_cache* c, int32_t layer, int32_t row0, int32_t n_rows,
+                              int64_t n) {
+  for (int b = row0; b < row0 + n_rows; ++b) {
+    const int64_t t = c->row_t(layer, b);
+    if (t < 0) return fail(HWKV_EINVAL, "layer %d row %d is idle (hwkv_reset_rows makes it active)", layer, b);
+    if (t + n > c->pol.max_ctx)
+      return fail(HWKV_ECAPACITY, "layer %d row %d: t=%lld + n=%lld exceeds max_ctx=%lld", layer, b,
+                  (long long)t, (long long)n, (long long)c->pol.max_ctx);
+  }
+  return HWKV_OK;
+}
+
+hwkv_status hwkv_append_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_t n_rows,
+                             const void* k, const void* v, int64_t n, void* cuda_stream) {
+  hwkv_status st = check_fresh(c, layer);
   if (st != HWKV_OK) return st;
+  if ((st = check_rows(c, row0, n_rows)) != HWKV_OK) return st;
   if (n < 0) return fail(HWKV_EINVAL, "n must be >= 0");
   if (n == 0) return ok();
   if (!k || !v) return fail(HWKV_EINVAL, "k/v is NULL");
-  if (c->t[layer] + n > c->pol.max_ctx)
-    return fail(HWKV_ECAPACITY, "layer %d: t=%lld + n=%lld exceeds max_ctx=%lld", layer,
-                (long long)c->t[layer], (long long)n, (long long)c->pol.max_ctx);
-  const AppendParams p = append_params(c, layer, k, v, n);
+  if ((st = check_room(c, layer, row0, n_rows, n)) != HWKV_OK) return st;
+  const AppendParams p = append_params(c, layer, row0, n_rows, k, v, n);
   cudaError_t e = launch_append(p, static_cast<cudaStream_t>(cuda_stream));
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "append launch: %s", cudaGetErrorString(e));
-  c->t[layer] += n;
+  for (int b = row0; b < row0 + n_rows; ++b) c->row_t(layer, b) += n;
   return ok();
 }
 
-hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void* k,
-                         const void* v, int64_t n, float scale, float* out, void* cuda_stream) {
-  hwkv_status st = check_layer(c, layer);
+hwkv_status hwkv_append(hwkv_cache* c, int32_t layer, const void* k, const void* v, int64_t n,
+                        void* cuda_stream) {
+  if (!c) return fail(HWKV_EINVAL, "cache is NULL");
+  return hwkv_append_rows(c, layer, 0, c->pol.batch, k, v, n, cuda_stream);
+}
+
+hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_t n_rows,
+                              const void* q, const void* k, const void* v, int64_t n, float scale,
+                              float* out, void* cuda_stream) {
+  hwkv_status st = check_fresh(c, layer);
   if (st != HWKV_OK) return st;
+  if ((st = check_rows(c, row0, n_rows)) != HWKV_OK) return st;
   if (n < 0) return fail(HWKV_EINVAL, "n must be >= 0");
   if (n == 0) return ok();
   if (!q || !k || !v || !out) return fail(HWKV_EINVAL, "q/k/v/out is NULL");
-  if (c->t[layer] + n > c->pol.max_ctx)
-    return fail(HWKV_ECAPACITY, "layer %d: t=%lld + n=%lld exceeds max_ctx=%lld", layer,
-                (long long)c->t[layer], (long long)n, (long long)c->pol.max_ctx);
+  if ((st = check_room(c, layer, row0, n_rows, n)) != HWKV_OK) return st;
+  const int64_t t_rows = c->row_t(layer, row0);
+  for (int b = row0 + 1; b < row0 + n_rows; ++b)
+    if (c->row_t(layer, b) != t_rows)
+      return fail(HWKV_EINVAL, "prefill rows must hold the same length (row %d: %lld, row %d: %lld)",
+                  row0, (long long)t_rows, b, (long long)c->row_t(layer, b));
   if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
   if (n > (int64_t)65535 * 16) return fail(HWKV_EUNSUPPORTED, "chunk of %lld tokens too long", (long long)n);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   PrefillParams p{};
   p.n_units = c->pol.n_kv_heads;
-  p.batch = c->pol.batch;
+  p.batch = n_rows;
+  p.row0 = row0;
   p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
   p.n_q_heads = c->pol.n_q_heads;
-  p.t0 = c->t[layer];
+  p.t0 = t_rows;
   p.n = n;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.q = static_cast<const __nv_bfloat16*>(q);
@@ -315,7 +407,7 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
   CUtensorMap q_map, ck_map, cv_map;
   {
     const cuuint64_t dim[3] = {(cuuint64_t)d, (cuuint64_t)c->pol.n_q_heads,
-                               (cuuint64_t)c->pol.batch * (cuuint64_t)n};
+                               (cuuint64_t)n_rows * (cuuint64_t)n};
     const cuuint64_t str[2] = {(cuuint64_t)d * 2, (cuuint64_t)c->pol.n_q_heads * d * 2};
     const cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)QP};
     CUresult r = encode(&q_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dim, str,
@@ -325,7 +417,7 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
   }
   {
     const cuuint64_t dim[3] = {(cuuint64_t)d, (cuuint64_t)c->pol.n_kv_heads,
-                               (cuuint64_t)c->pol.batch * (cuuint64_t)n};
+                               (cuuint64_t)n_rows * (cuuint64_t)n};
     const cuuint64_t str[2] = {(cuuint64_t)d * 2, (cuuint64_t)c->pol.n_kv_heads * d * 2};
     const cuuint32_t box[3] = {64, 1, 64};
     CUresult r = encode(&ck_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(k), dim,
@@ -337,140 +429,165 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(HWKV_EINVAL, "k/v tensor map rejected (%d): k/v must be 16-byte aligned", (int)r);
   }
-  if ((int64_t)c->pol.batch * n + 128 >= (int64_t)INT32_MAX)
+  if ((int64_t)n_rows * n + 128 >= (int64_t)INT32_MAX)
     return fail(HWKV_EUNSUPPORTED, "batch x chunk exceeds the TMA coordinate range");
   cudaError_t e = launch_prefill_tc(p, d, q_map, ck_map, cv_map, c->kv_map, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "prefill launch: %s", cudaGetErrorString(e));
   // attend first, then write the chunk's retained tokens (stream order)
-  const AppendParams ap = append_params(c, layer, k, v, n);
+  const AppendParams ap = append_params(c, layer, row0, n_rows, k, v, n);
   e = launch_append(ap, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "append launch: %s", cudaGetErrorString(e));
-  c->t[layer] += n;
+  for (int b = row0; b < row0 + n_rows; ++b) c->row_t(layer, b) += n;
   return ok();
 }
 
-// Decode tile plan: equal-length tiles (multiple of 64 tokens) over every
-// (batch row, KV head) ring. The length is chosen to balance the persistent
-// grid: minimise (tiles per CTA) x (tile length + a fixed per-tile cost).
-static void plan_decode(const hwkv_cache* c, int32_t layer, int max_tiles, DecodeParams& p,
-                        int& grid, int64_t t) {
-  const int H = c->pol.n_kv_heads, B = c->pol.batch;
-  int64_t n_valid[kMaxKvHeads];
-  int64_t longest = 0;
-  for (int h = 0; h < H; ++h) {
-    const Unit& u = c->lay.units[(size_t)layer * H + h];
-    n_valid[h] = std::min(t, u.cap);
-    longest = std::max(longest, n_valid[h]);
-  }
+hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void* k,
+                         const void* v, int64_t n, float scale, float* out, void* cuda_stream) {
+  if (!c) return fail(HWKV_EINVAL, "cache is NULL");
+  return hwkv_prefill_rows(c, layer, 0, c->pol.batch, q, k, v, n, scale, out, cuda_stream);
+}
+
+// CTAs of a decode split launch. A grid of one (shared-memory-filling) CTA on
+// every SM cannot start until every SM is free, and leaves no room for the
+// combine kernel's CTAs to become resident ahead of time; measured on GB300 that
+// costs ~7 us per launch, more than 8 extra SMs gain below ~1 GB of K/V per
+// layer-step. So small steps leave 8 SMs free. `tokens` = resident K/V rows the
+// step reads (an estimate is enough: it changes speed, not results).
+static int decode_grid_cap(const hwkv_cache* c, int64_t tokens) {
   const int sms = std::max(1, c->num_sms);
-  auto count = [&](int64_t len) {
-    int64_t n = 0;
-    for (int h = 0; h < H; ++h) n += (n_valid[h] + len - 1) / len;
-    return n * B;
-  };
-  const int64_t per_tile_cost = 96;  // tokens-equivalent of a tile's fixed cost
-  int64_t best_len = 0;
-  double best = 0;
-  const int64_t max_len = std::max<int64_t>(64, (longest + 63) / 64 * 64);
-  for (int64_t len = 128; ; len = len < 1024 ? len + 64 : len + len / 8 / 64 * 64) {
-    const int64_t L = std::min(len, max_len);
-    const int64_t nt = count(L);
-    if (nt <= max_tiles) {
-      const int64_t g = std::min<int64_t>(nt, sms);
-      const double cost = (double)((nt + g - 1) / g) * (double)(L + per_tile_cost);
-      if (best_len == 0 || cost < best) {
-        best = cost;
-        best_len = L;
-      }
-    }
-    if (L >= max_len) break;
+  const int64_t bytes = tokens * 4 * c->pol.head_dim;
+  constexpr int64_t kFullGridBytes = 1LL << 30;
+  return (bytes >= kFullGridBytes || sms <= 16) ? sms : sms - 8;
+}
+
+// resident K/V rows a step of `layer` reads, from the host copy of the lengths
+static int64_t step_tokens(const hwkv_cache* c, int32_t layer, int add) {
+  const int H = c->pol.n_kv_heads;
+  int64_t n = 0;
+  for (int b = 0; b < c->pol.batch; ++b) {
+    const int64_t t = c->row_t(layer, b);
+    if (t < 0) continue;
+    for (int h = 0; h < H; ++h) n += std::min(t + add, c->lay.units[(size_t)layer * H + h].cap);
   }
-  if (best_len == 0) best_len = max_len;
-  p.tile_len = (int32_t)best_len;
-  int32_t begin = 0;
-  for (int h = 0; h < H; ++h) {
-    const Unit& u = c->lay.units[(size_t)layer * H + h];
-    DecodeUnit& du = p.u[h];
-    du.k_row0 = u.k_row0;
-    du.v_row0 = u.v_row0;
-    du.cap = u.cap;
-    du.n_valid = (int32_t)n_valid[h];
-    du.n_tiles = (int32_t)((n_valid[h] + best_len - 1) / best_len);
-    du.tile_begin = begin;
-    du.s_new = (int32_t)((t - 1) % u.cap);  // slot of the newest token (fused step)
-    begin += du.n_tiles;
+  return n;
+}
+
+enum DecodeMode { kPlain = 0, kFused = 1, kFusedGraph = 2 };
+
+// the fields of a ring-mode decode launch that do not depend on the call's tensors
+static void ring_params(const hwkv_cache* c, int32_t layer, DecodeParams& p, int lens_inc) {
+  p.n_units = c->pol.n_kv_heads;
+  p.batch = c->pol.batch;
+  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
+  p.n_q_heads = c->pol.n_q_heads;
+  p.err = c->err();
+  p.lens = c->lens(layer);
+  p.lens_inc = lens_inc;
+  p.max_ctx = c->pol.max_ctx;
+  // a segment's fixed cost (query load, merge, partial write) ~ the time to stream
+  // 256 KB of K/V at one CTA's share of HBM bandwidth, in 64-key stages
+  p.seg_cost = std::max(1, (256 << 10) / (4 * c->pol.head_dim) / kStageTokens);
+  for (int h = 0; h < p.n_units; ++h) {
+    const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
+    p.u[h] = DecodeUnit{u.k_row0, u.v_row0, u.cap};
   }
-  p.tiles_per_b = begin;
-  p.n_tiles = begin * B;
-  // per-ring tiles are bounded by max_tiles / batch <= max(2048, 2 * n_kv_heads) < kCombineMaxTiles
-  grid = std::min(p.n_tiles, sms);
+}
+
+// One decode call of a layer: the split kernel plans its work on the GPU from
+// the device lengths (so one launch serves uniform, ragged and idle rows, and
+// replays correctly from a CUDA graph), then the combine kernel merges.
+static hwkv_status decode_call(hwkv_cache* c, int32_t layer, const void* q, const void* k_new,
+                               const void* v_new, float scale, float* out, void* cuda_stream,
+                               DecodeMode mode) {
+  hwkv_status st = mode == kFusedGraph ? check_layer(c, layer) : check_fresh(c, layer);
+  if (st != HWKV_OK) return st;
+  if (!q || !out) return fail(HWKV_EINVAL, "q/out is NULL");
+  if (mode != kPlain && (!k_new || !v_new)) return fail(HWKV_EINVAL, "k_new/v_new is NULL");
+  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
+  const int B = c->pol.batch;
+  if (mode == kPlain) {
+    bool any = false;
+    for (int b = 0; b < B; ++b) any |= c->row_t(layer, b) > 0;
+    if (!any) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
+  } else if (mode == kFused) {
+    for (int b = 0; b < B; ++b)
+      if (c->row_t(layer, b) + 1 > c->pol.max_ctx)
+        return fail(HWKV_ECAPACITY, "layer %d row %d: t=%lld + 1 exceeds max_ctx=%lld", layer, b,
+                    (long long)c->row_t(layer, b), (long long)c->pol.max_ctx);
+  }
+  DecodeParams p{};
+  ring_params(c, layer, p, mode == kPlain ? 0 : 1);
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.part_o = c->part_o();
+  p.part_ml = c->part_ml();
+  p.out = out;
+  p.plan = c->plan();
+  if (mode != kPlain) {
+    p.k_new = static_cast<const __nv_bfloat16*>(k_new);
+    p.v_new = static_cast<const __nv_bfloat16*>(v_new);
+    p.arena = c->k_base();
+  }
+  // the host copy of the lengths sizes the grid (stale under graph capture: an estimate)
+  const int grid = decode_grid_cap(c, step_tokens(c, layer, mode == kPlain ? 0 : 1));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
+  e = launch_decode_combine(p, c->pol.head_dim, s);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
+  if (mode == kFused)
+    for (int b = 0; b < B; ++b)
+      if (c->row_t(layer, b) >= 0) c->row_t(layer, b) += 1;
+  if (mode == kFusedGraph) c->dev_owned[layer] = 1;
+  return ok();
 }
 
 hwkv_status hwkv_decode_attn(hwkv_cache* c, int32_t layer, const void* q, float scale, float* out,
                              void* cuda_stream) {
-  hwkv_status st = check_layer(c, layer);
-  if (st != HWKV_OK) return st;
-  if (!q || !out) return fail(HWKV_EINVAL, "q/out is NULL");
-  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
-  if (c->t[layer] <= 0) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
-  if (c->t[layer] > INT32_MAX) return fail(HWKV_EUNSUPPORTED, "ring longer than 2^31");
-  DecodeParams p{};
-  p.n_units = c->pol.n_kv_heads;
-  p.batch = c->pol.batch;
-  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
-  p.n_q_heads = c->pol.n_q_heads;
-  p.scale_log2 = scale * 1.4426950408889634f;
-  p.q = static_cast<const __nv_bfloat16*>(q);
-  p.part_o = c->part_o();
-  p.part_ml = c->part_ml();
-  p.out = out;
-  p.err = c->err();
-  int grid = 0;
-  plan_decode(c, layer, c->lay.max_tiles, p, grid, c->t[layer]);
-  if (p.n_tiles > c->lay.max_tiles)
-    return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
-  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s);
-  if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
-  e = launch_decode_combine(p, c->pol.head_dim, s);
-  if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
-  return ok();
+  return decode_call(c, layer, q, nullptr, nullptr, scale, out, cuda_stream, kPlain);
 }
 
 hwkv_status hwkv_decode_step(hwkv_cache* c, int32_t layer, const void* q, const void* k_new,
                              const void* v_new, float scale, float* out, void* cuda_stream) {
-  hwkv_status st = check_layer(c, layer);
-  if (st != HWKV_OK) return st;
-  if (!q || !out || !k_new || !v_new) return fail(HWKV_EINVAL, "q/k_new/v_new/out is NULL");
-  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
-  if (c->t[layer] + 1 > c->pol.max_ctx)
-    return fail(HWKV_ECAPACITY, "layer %d: t=%lld + 1 exceeds max_ctx=%lld", layer,
-                (long long)c->t[layer], (long long)c->pol.max_ctx);
-  if (c->t[layer] + 1 > INT32_MAX) return fail(HWKV_EUNSUPPORTED, "ring longer than 2^31");
-  DecodeParams p{};
-  p.n_units = c->pol.n_kv_heads;
-  p.batch = c->pol.batch;
-  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
-  p.n_q_heads = c->pol.n_q_heads;
-  p.scale_log2 = scale * 1.4426950408889634f;
-  p.q = static_cast<const __nv_bfloat16*>(q);
-  p.part_o = c->part_o();
-  p.part_ml = c->part_ml();
-  p.out = out;
-  p.err = c->err();
-  p.k_new = static_cast<const __nv_bfloat16*>(k_new);
-  p.v_new = static_cast<const __nv_bfloat16*>(v_new);
-  p.arena = c->k_base();
-  int grid = 0;
-  plan_decode(c, layer, c->lay.max_tiles, p, grid, c->t[layer] + 1);  // state after the append
-  if (p.n_tiles > c->lay.max_tiles)
-    return fail(HWKV_EUNSUPPORTED, "decode plan needs %d tiles > %d", p.n_tiles, c->lay.max_tiles);
+  return decode_call(c, layer, q, k_new, v_new, scale, out, cuda_stream, kFused);
+}
+
+hwkv_status hwkv_decode_step_graph(hwkv_cache* c, int32_t layer, const void* q, const void* k_new,
+                                   const void* v_new, float scale, float* out, void* cuda_stream) {
+  return decode_call(c, layer, q, k_new, v_new, scale, out, cuda_stream, kFusedGraph);
+}
+
+hwkv_status hwkv_sync_lens(hwkv_cache* c, void* cuda_stream) {
+  if (!c) return fail(HWKV_EINVAL, "cache is NULL");
+  const size_t n = (size_t)c->pol.n_layers * c->pol.batch;
+  std::vector<int32_t> host(n);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s);
-  if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
-  e = launch_decode_combine(p, c->pol.head_dim, s);
-  if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
-  c->t[layer] += 1;
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess) e = cudaMemcpy(host.data(), c->lens(0), n * 4, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "length copy: %s", cudaGetErrorString(e));
+  for (size_t i = 0; i < n; ++i) c->t[i] = host[i] < 0 ? -1 : host[i];
+  return ok();
+}
+
+hwkv_status hwkv_reset_rows(hwkv_cache* c, int32_t row0, int32_t n_rows, int32_t idle,
+                            void* cuda_stream) {
+  if (!c) return fail(HWKV_EINVAL, "cache is NULL");
+  hwkv_status st = check_rows(c, row0, n_rows);
+  if (st != HWKV_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  for (int l = 0; l < c->pol.n_layers; ++l) {
+    cudaError_t e = cudaMemsetAsync(c->lens(l) + row0, idle ? 0xFF : 0, (size_t)n_rows * 4, s);
+    if (e != cudaSuccess) return fail(HWKV_ECUDA, "length reset: %s", cudaGetErrorString(e));
+    for (int b = row0; b < row0 + n_rows; ++b) c->row_t(l, b) = idle ? -1 : 0;
+  }
+  return ok();
+}
+
+hwkv_status hwkv_row_len(const hwkv_cache* c, int32_t layer, int32_t row, int64_t* t) {
+  hwkv_status st = check_fresh(c, layer);
+  if (st != HWKV_OK) return st;
+  if (row < 0 || row >= c->pol.batch || !t) return fail(HWKV_EINVAL, "bad row or NULL t");
+  *t = c->row_t(layer, row);
   return ok();
 }
 
@@ -482,9 +599,12 @@ hwkv_status hwkv_residency_bytes(const hwkv_cache* c, int32_t layer, uint64_t* b
   uint64_t total = 0;
   for (int l = 0; l < c->pol.n_layers; ++l) {
     if (layer >= 0 && l != layer) continue;
+    hwkv_status st = refresh_lens(c, l);
+    if (st != HWKV_OK) return st;
     for (int h = 0; h < H; ++h) {
       const Unit& u = c->lay.units[(size_t)l * H + h];
-      total += (uint64_t)std::min(c->t[l], u.cap) * per_token * (uint64_t)c->pol.batch;
+      for (int b = 0; b < c->pol.batch; ++b)  // idle rows (-1) hold nothing
+        total += (uint64_t)std::min(std::max<int64_t>(c->row_t(l, b), 0), u.cap) * per_token;
     }
   }
   *bytes = total;
@@ -507,10 +627,12 @@ hwkv_status hwkv_allocated_ring_bytes(const hwkv_cache* c, int32_t layer, uint64
 }
 
 hwkv_status hwkv_seq_len(const hwkv_cache* c, int32_t layer, int64_t* t) {
-  hwkv_status st = check_layer(c, layer);
+  hwkv_status st = check_fresh(c, layer);
   if (st != HWKV_OK) return st;
   if (!t) return fail(HWKV_EINVAL, "t is NULL");
-  *t = c->t[layer];
+  if (!c->uniform(layer, t))
+    return fail(HWKV_EINVAL, "layer %d rows hold different lengths (or are idle): use hwkv_row_len",
+                layer);
   return ok();
 }
 
@@ -549,7 +671,8 @@ hwkv_status hwkv_sync_check(hwkv_cache* c) {
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "sync: %s", cudaGetErrorString(e));
   if (word != 0) {
     cudaMemset(c->err(), 0, sizeof(int));
-    return fail(HWKV_EKERNEL, "kernel error word 0x%x (1 = bounded wait gave up, 2 = bad index)",
+    return fail(HWKV_EKERNEL, "kernel error word 0x%x (1 = bounded wait gave up, 2 = bad index, "
+                "4 = a graph-mode step skipped a row at max_ctx)",
                 word);
   }
   return ok();
@@ -596,22 +719,22 @@ static void* static_scratch_address(int device, cudaError_t* err) {
 
 hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q, float scale,
                                     float* out, void* cuda_stream) {
-  hwkv_status st = check_layer(c, layer);
+  hwkv_status st = check_fresh(c, layer);
   if (st != HWKV_OK) return st;
   if (!q || !out) return fail(HWKV_EINVAL, "q/out is NULL");
-  if (c->t[layer] <= 0) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
-  if (c->t[layer] > INT32_MAX) return fail(HWKV_EUNSUPPORTED, "ring longer than 2^31");
+  if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
+  bool any = false;
+  for (int b = 0; b < c->pol.batch; ++b) any |= c->row_t(layer, b) > 0;
+  if (!any) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
   const int d = c->pol.head_dim;
-  const size_t o_bytes_per_tile = (size_t)kMaxGroup * d * 4;
-  const size_t ml_bytes_per_tile = (size_t)kMaxGroup * 8;
-  const int cap_tiles =
-      (int)((HWKV_DECODE_STATIC_SCRATCH_BYTES - kAlign) / (o_bytes_per_tile + ml_bytes_per_tile));
-  const int min_tiles = c->pol.batch * c->pol.n_kv_heads;  // one tile per (batch row, KV head)
-  if (min_tiles > cap_tiles)
-    return fail(HWKV_EINVAL,
-                "batch x n_kv_heads = %d exceeds the %d tiles the %d-byte static decode scratch "
-                "holds at head_dim %d",
-                min_tiles, cap_tiles, (int)HWKV_DECODE_STATIC_SCRATCH_BYTES, d);
+  const int grid = decode_grid_cap(c, step_tokens(c, layer, 0));
+  // two partial slots per CTA, then the plan table
+  const size_t o_bytes = align_up((size_t)2 * grid * kMaxGroup * d * 4, kAlign);
+  const size_t ml_bytes = align_up((size_t)2 * grid * kMaxGroup * 8, kAlign);
+  const size_t plan_bytes = (size_t)(4 + 2 * c->pol.batch * c->pol.n_kv_heads) * 8;
+  if (o_bytes + ml_bytes + plan_bytes > HWKV_DECODE_STATIC_SCRATCH_BYTES)
+    return fail(HWKV_EINVAL, "static decode needs %zu scratch bytes > %u", o_bytes + ml_bytes + plan_bytes,
+                (unsigned)HWKV_DECODE_STATIC_SCRATCH_BYTES);
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
@@ -620,21 +743,13 @@ hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q,
     return fail(HWKV_ECUDA, "cudaGetSymbolAddress(static decode scratch) on device %d: %s", dev,
                 cudaGetErrorString(e));
   DecodeParams p{};
-  p.n_units = c->pol.n_kv_heads;
-  p.batch = c->pol.batch;
-  p.group = c->pol.n_q_heads / c->pol.n_kv_heads;
-  p.n_q_heads = c->pol.n_q_heads;
+  ring_params(c, layer, p, 0);
   p.scale_log2 = scale * 1.4426950408889634f;
   p.q = static_cast<const __nv_bfloat16*>(q);
   p.part_o = reinterpret_cast<float*>(scratch);
-  p.part_ml = reinterpret_cast<float2*>(scratch + align_up((size_t)cap_tiles * o_bytes_per_tile, kAlign));
+  p.part_ml = reinterpret_cast<float2*>(scratch + o_bytes);
+  p.plan = reinterpret_cast<int64_t*>(scratch + o_bytes + ml_bytes);
   p.out = out;
-  p.err = c->err();
-  int grid = 0;
-  plan_decode(c, layer, cap_tiles, p, grid, c->t[layer]);
-  if (p.n_tiles > cap_tiles)
-    return fail(HWKV_EINVAL, "decode plan needs %d tiles > %d in the static scratch", p.n_tiles,
-                cap_tiles);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   e = launch_decode(p, c->kv_map, c->kv_map, d, grid, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
@@ -779,7 +894,6 @@ hwkv_status hwkv_calib_scores(const hwkv_calib_desc* d, const void* q, const voi
   p.err = reinterpret_cast<int*>(ws + P.off_err);
   p.tiles = reinterpret_cast<const CalibTile*>(ws + P.off_tiles);
   p.n_tiles = (int32_t)P.tiles.size();
-  p.tiles_per_b = p.n_tiles;
   if (p.n_tiles > 0) {
     e = launch_decode(p, kmap, vmap, D, std::min(p.n_tiles, std::max(1, sms)), s);
     if (e != cudaSuccess) return fail(HWKV_ECUDA, "calib tile launch: %s", cudaGetErrorString(e));

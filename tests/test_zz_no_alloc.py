@@ -12,6 +12,7 @@ makes pytest collect it last.
 import numpy as np
 import pytest
 
+import hwkv_gen
 import paper_2609_02029_gb300 as hwkv
 from harness import Run, assert_close
 
@@ -41,19 +42,20 @@ def test_static_scratch_decode_matches_allocating_decode():
         r.close()
 
 
-def test_static_scratch_rejects_sizes_beyond_its_maximum():
+def test_static_scratch_serves_the_largest_batches():
     import torch
-    # 256 batch rows x 4 KV heads = 1024 (row, head) pairs > 508 tiles at head_dim 256
-    r = Run(1, 256, 8, 4, 256, 8, [0, 4, 0, 2])
+    # 256 batch rows x 4 KV heads: the work plan and partials (two per CTA) still fit
+    r = Run(1, 256, 8, 4, 256, 300, [0, 4, 0, 64], seed=4)
     try:
-        r.append(0, 1)
-        q = torch.zeros((256, 8, 256), dtype=torch.bfloat16, device="cuda")
-        out = torch.empty((256, 8, 256), dtype=torch.float32, device="cuda")
-        with pytest.raises(hwkv.HwkvError) as e:
-            hwkv.hwkv_decode_attn_static(r.cache, 0, q, 1.0, out, r.stream)
-        assert e.value.status == hwkv.HWKV_EINVAL
-        assert "static decode scratch" in hwkv.hwkv_last_error()
-        hwkv.hwkv_decode_attn(r.cache, 0, q, 1.0, out, r.stream)  # the allocating path still works
-        hwkv.hwkv_sync_check(r.cache)
+        r.fill(0, 200)
+        q = r.gen(hwkv_gen.Q, 0, 199, 1, r.Hq).view(r.B, r.Hq, r.d)
+        ref = torch.empty((256, 8, 256), dtype=torch.float32, device="cuda")
+        got = torch.empty_like(ref)
+        hwkv.hwkv_decode_attn(r.cache, 0, q, r.scale, ref, r.stream)
+        for _ in range(2):
+            hwkv.hwkv_decode_attn_static(r.cache, 0, q, r.scale, got, r.stream)
+            hwkv.hwkv_sync_check(r.cache)
+            assert_close(got.cpu().numpy(), ref.cpu().numpy().astype(np.float64),
+                         "static vs allocating decode, 256 rows")
     finally:
         r.close()
