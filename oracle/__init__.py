@@ -73,6 +73,23 @@ def lib():
         L.oracle_budget_select.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
                                            ctypes.c_double]
         L.oracle_budget_select.restype = ctypes.c_int64
+        L.oracle_e4m3_decode.argtypes = [ctypes.c_uint8]
+        L.oracle_e4m3_decode.restype = ctypes.c_double
+        L.oracle_e4m3_encode.argtypes = [ctypes.c_float]
+        L.oracle_e4m3_encode.restype = ctypes.c_uint8
+        L.oracle_quantize_row_e4m3.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p,
+                                               ctypes.c_void_p]
+        L.oracle_quantize_row_e4m3.restype = ctypes.c_int
+        L.oracle_window_attention_fp8.argtypes = [
+            ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64,
+            ctypes.c_int64, ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p]
+        L.oracle_window_attention_fp8.restype = ctypes.c_int
+        L.oracle_ring_expected_fp8_gen.argtypes = [
+            ctypes.POINTER(GenDesc), ctypes.c_uint32, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
+            ctypes.c_void_p]
+        L.oracle_ring_expected_fp8_gen.restype = ctypes.c_int
         _lib = L
     return _lib
 
@@ -216,3 +233,72 @@ def budget_select(beta, phi, budget):
     b = np.ascontiguousarray(beta, dtype=np.float64)
     f = np.ascontiguousarray(phi, dtype=np.float64)
     return int(lib().oracle_budget_select(_p(b), _p(f), len(b), float(budget)))
+
+
+# ---------------------------------------------------------------- 8-bit format
+# The cache format p_KV of Sec. 3.1 with 8-bit keys and values: E4M3 codes and one
+# fp32 scale per stored row (a reading; the paper names no 8-bit format).
+
+def e4m3_decode(code):
+    """Value of an E4M3 code (exact; NaN for S.1111.111)."""
+    return float(lib().oracle_e4m3_decode(int(code)))
+
+
+def e4m3_encode(x):
+    """Nearest E4M3 code of the float32 x (ties to even, |x| > 448 -> 448, NaN -> 0x7F)."""
+    return int(lib().oracle_e4m3_encode(float(np.float32(x))))
+
+
+def quantize_row_e4m3(x_bf16):
+    """One stored row: bf16 bits [d] -> (codes uint8 [d], scale float32)."""
+    x = np.ascontiguousarray(x_bf16, dtype=np.uint16)
+    codes = np.zeros(len(x), dtype=np.uint8)
+    scale = np.zeros(1, dtype=np.float32)
+    if lib().oracle_quantize_row_e4m3(_p(x), len(x), _p(codes), _p(scale)) != 0:
+        raise ValueError("bad row")
+    return codes, np.float32(scale[0])
+
+
+def quantize_rows_e4m3(X_bf16):
+    """Rows [n][d] of bf16 bits -> (codes [n][d], scales [n])."""
+    X = np.ascontiguousarray(X_bf16, dtype=np.uint16)
+    codes = np.zeros(X.shape, dtype=np.uint8)
+    scales = np.zeros(X.shape[0], dtype=np.float32)
+    for r in range(X.shape[0]):
+        codes[r], scales[r] = quantize_row_e4m3(X[r])
+    return codes, scales
+
+
+def dequantize_rows_e4m3(codes, scales):
+    """decode(code) * scale, in float64."""
+    table = np.array([e4m3_decode(c) for c in range(256)])
+    return table[np.asarray(codes)] * np.asarray(scales, dtype=np.float64)[:, None]
+
+
+def window_attention_fp8(Q, pos, Kc, Ks, Vc, Vs, W, gamma):
+    """Window attention (Sec. 3.2) over a history stored in the 8-bit format:
+    Q bf16 bits [R][d]; Kc/Vc codes [T][d]; Ks/Vs scales [T]. Returns (O [R][d], sum_pi)."""
+    Q = np.ascontiguousarray(Q, dtype=np.uint16)
+    Kc = np.ascontiguousarray(Kc, dtype=np.uint8)
+    Vc = np.ascontiguousarray(Vc, dtype=np.uint8)
+    Ks = np.ascontiguousarray(Ks, dtype=np.float32)
+    Vs = np.ascontiguousarray(Vs, dtype=np.float32)
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    R, d = Q.shape
+    O = np.zeros((R, d))
+    sp = np.zeros(R)
+    rc = lib().oracle_window_attention_fp8(_p(Q), d, _p(pos), R, _p(Kc), _p(Ks), _p(Vc), _p(Vs),
+                                           Kc.shape[0], d, int(W), float(gamma), _p(O), _p(sp))
+    if rc != 0:
+        raise ValueError("oracle_window_attention_fp8 failed (%d)" % rc)
+    return O, sp
+
+
+def ring_expected_fp8_gen(g, tensor, layer, b, kvh, d, t, cap):
+    """Expected 8-bit ring after positions 0..t-1: (codes [cap][d], scales [cap])."""
+    codes = np.zeros((cap, d), dtype=np.uint8)
+    scales = np.zeros(cap, dtype=np.float32)
+    if lib().oracle_ring_expected_fp8_gen(ctypes.byref(g), tensor, layer, b, kvh, d, t, cap,
+                                          _p(codes), _p(scales)) != 0:
+        raise ValueError("bad ring arguments")
+    return codes, scales

@@ -27,6 +27,16 @@
  *                       (Eq. threshold-selection), budget selector (App. A.2,
  *                       Eq. budget-selector).
  *
+ *   - 8-bit cache format (p_KV of Sec. 3.1; the paper names no 8-bit format, so
+ *                       this is a reading): E4M3 codes (1 sign bit, 4 exponent bits
+ *                       with bias 7, 3 mantissa bits, no infinities, S.1111.111 =
+ *                       NaN, largest finite 448) with one fp32 scale per stored row
+ *                       (one token of one KV head): s = amax / 448, code = nearest
+ *                       E4M3 value of x / s (ties to even, beyond 448 clamped to 448),
+ *                       dequantised value decode(code) * s. Attention over such a
+ *                       cache reads the dequantised rows (Sec. 3.1: when the format
+ *                       changes execution, every compared output uses it).
+ *
  * Windows are int64: 0 (HWKV_WINDOW_FULL) means full history; any W >= the
  * context is equivalent to full (Sec. 3.1). bf16 inputs are widened exactly to
  * double. Row loops may run under OpenMP; each row is computed independently.
@@ -242,6 +252,143 @@ int oracle_ring_expected_gen(const hwkv_gen_desc* g, uint32_t tensor, int32_t la
                                    : hwkv_gen_elem(g, tensor, (uint32_t)layer, (uint32_t)b,
                                                    (uint32_t)kvh, (uint64_t)pos[j], (uint32_t)i, s);
   free(pos);
+  return 0;
+}
+
+/* ------------------------------------------------------- 8-bit KV format */
+
+/* value of an E4M3 code, from its bit fields (exact; NaN for S.1111.111) */
+double oracle_e4m3_decode(uint8_t c) {
+  const int sign = c >> 7, e = (c >> 3) & 15, m = c & 7;
+  if (e == 15 && m == 7) return NAN;
+  const double mag = e == 0 ? ldexp((double)m / 8.0, -6)               /* subnormal */
+                            : ldexp(1.0 + (double)m / 8.0, e - 7);     /* normal */
+  return sign ? -mag : mag;
+}
+
+/*
+ * Nearest E4M3 code of x: the finite magnitudes (codes 0x00 .. 0x7E, increasing
+ * with the code) are searched for the two that bracket |x|; the nearer one wins,
+ * a tie goes to the even code (mantissa lsb 0); |x| above 448, including
+ * infinity, clamps to 448; NaN gives 0x7F. The sign bit is x's sign bit.
+ */
+uint8_t oracle_e4m3_encode(float x) {
+  if (isnan(x)) return 0x7F;
+  const uint8_t sign = signbit(x) ? 0x80 : 0x00;
+  const double a = fabs((double)x);
+  if (a >= 448.0) return (uint8_t)(sign | 0x7E);
+  uint8_t lo = 0;
+  for (uint8_t c = 1; c <= 0x7E; ++c)
+    if (oracle_e4m3_decode(c) <= a) lo = c;
+  /* a < 448 here, so lo < 0x7E and lo + 1 is the next larger magnitude */
+  const uint8_t hi = (uint8_t)(lo + 1);
+  const double dlo = a - oracle_e4m3_decode(lo), dhi = oracle_e4m3_decode(hi) - a;
+  uint8_t c;
+  if (dlo < dhi) c = lo;
+  else if (dhi < dlo) c = hi;
+  else c = (lo & 1) ? hi : lo;
+  return (uint8_t)(sign | c);
+}
+
+/*
+ * One stored row in the 8-bit format: x[d] (bf16 bits) -> codes[d], *scale.
+ * amax = max |x_i|; s = amax / 448 in float arithmetic; code_i = encode(x_i / s)
+ * with x_i / s a float division; amax = 0 gives s = 0 and all-zero codes.
+ */
+int oracle_quantize_row_e4m3(const uint16_t* x, int64_t d, uint8_t* codes, float* scale) {
+  if (d <= 0) return 1;
+  float amax = 0.0f;
+  for (int64_t i = 0; i < d; ++i) {
+    const float v = (float)fabs(bf16_to_double(x[i]));
+    if (v > amax) amax = v;
+  }
+  if (amax == 0.0f) {
+    for (int64_t i = 0; i < d; ++i) codes[i] = 0;
+    *scale = 0.0f;
+    return 0;
+  }
+  const volatile float s = amax / 448.0f;
+  for (int64_t i = 0; i < d; ++i) {
+    const volatile float y = (float)bf16_to_double(x[i]) / s;
+    codes[i] = oracle_e4m3_encode(y);
+  }
+  *scale = s;
+  return 0;
+}
+
+static double dequant(uint8_t c, float s) { return oracle_e4m3_decode(c) * (double)s; }
+
+/*
+ * oracle_window_attention_bf16 over a cache in the 8-bit format: key/value row
+ * s of the history is decode(codes[s][i]) * scale[s]. Kc/Vc [T][d] codes,
+ * Ks/Vs [T] scales, indexed by absolute position.
+ */
+int oracle_window_attention_fp8(const uint16_t* Q, int64_t ldq, const int64_t* pos, int64_t R,
+                                const uint8_t* Kc, const float* Ks, const uint8_t* Vc,
+                                const float* Vs, int64_t T, int64_t d, int64_t W, double gamma,
+                                double* O, double* sum_pi) {
+  if (R < 0 || d <= 0 || W < 0) return 1;
+  for (int64_t r = 0; r < R; ++r)
+    if (pos[r] < 0 || pos[r] >= T) return 1;
+  int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t r = 0; r < R; ++r) {
+    const int64_t p = pos[r];
+    const int64_t lo = oracle_window_lo(p, W);
+    const int64_t n = p - lo + 1;
+    double* q = (double*)malloc(sizeof(double) * (size_t)d);
+    double* K = (double*)malloc(sizeof(double) * (size_t)(n * d));
+    double* V = (double*)malloc(sizeof(double) * (size_t)(n * d));
+    if (!q || !K || !V) {
+      bad = 1;
+    } else {
+      for (int64_t i = 0; i < d; ++i) q[i] = bf16_to_double(Q[r * ldq + i]);
+      for (int64_t s = lo; s <= p; ++s)
+        for (int64_t i = 0; i < d; ++i) {
+          K[(s - lo) * d + i] = dequant(Kc[s * d + i], Ks[s]);
+          V[(s - lo) * d + i] = dequant(Vc[s * d + i], Vs[s]);
+        }
+      double sp = oracle_attend(q, K, V, n, d, gamma, O + r * d, NULL);
+      if (sum_pi) sum_pi[r] = sp;
+    }
+    free(q);
+    free(K);
+    free(V);
+  }
+  return bad ? 2 : 0;
+}
+
+/*
+ * Expected ring in the 8-bit format for one (layer, batch row, KV head) after
+ * positions 0..t-1: slot j holds the quantised generated row of the position
+ * it holds (codes[j][d], scale[j]); zeros where no position is held.
+ */
+int oracle_ring_expected_fp8_gen(const hwkv_gen_desc* g, uint32_t tensor, int32_t layer,
+                                 int32_t b, int32_t kvh, int32_t d, int64_t t, int64_t cap,
+                                 uint8_t* codes, float* scales) {
+  if (!g || cap <= 0 || t < 0 || d <= 0) return 1;
+  int64_t* pos = (int64_t*)malloc(sizeof(int64_t) * (size_t)cap);
+  uint16_t* row = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)d);
+  if (!pos || !row) {
+    free(pos);
+    free(row);
+    return 2;
+  }
+  oracle_ring_positions(t, cap, pos);
+  const float hs = hwkv_gen_head_scale(g, tensor, (uint32_t)layer, (uint32_t)kvh);
+  for (int64_t j = 0; j < cap; ++j) {
+    if (pos[j] < 0) {
+      memset(codes + j * d, 0, (size_t)d);
+      scales[j] = 0.0f;
+      continue;
+    }
+    for (int32_t i = 0; i < d; ++i)
+      row[i] = hwkv_gen_elem(g, tensor, (uint32_t)layer, (uint32_t)b, (uint32_t)kvh,
+                             (uint64_t)pos[j], (uint32_t)i, hs);
+    oracle_quantize_row_e4m3(row, d, codes + j * d, scales + j);
+  }
+  free(pos);
+  free(row);
   return 0;
 }
 
