@@ -151,22 +151,28 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------ GPU decode
-def decode_bytes(wl, max_ctx, t):
+def token_bytes(wl, fp8=False):
+    """Bytes one resident token of one KV head occupies: K and V rows in bf16, or
+    E4M3 codes plus a 4-byte scale per row."""
+    return 2 * (wl.head_dim + 4) if fp8 else 4 * wl.head_dim
+
+
+def decode_bytes(wl, max_ctx, t, fp8=False):
     """Algorithmic bytes of one decode launch per layer at length t: every
-    resident K/V row read once, batch x sum_h min(t, cap_h) x 4 d (q and out
-    are under 0.1 % and excluded)."""
+    resident K/V row read once, batch x sum_h min(t, cap_h) x token_bytes (q and
+    out are under 0.1 % and excluded)."""
     per_layer = []
     for layer in range(wl.n_layers):
         s = 0
         for h in range(wl.n_kv_heads):
             W = wl.windows[layer * wl.n_kv_heads + h]
             cap = max_ctx if (W == 0 or W >= max_ctx) else W
-            s += wl.batch * min(t, cap) * 4 * wl.head_dim
+            s += wl.batch * min(t, cap) * token_bytes(wl, fp8)
         per_layer.append(s)
     return per_layer
 
 
-def run_gpu(args, wl, world, rank, local):
+def run_gpu(args, wl, world, rank, local, fp8=False):
     import torch
 
     import hwkv_gen
@@ -186,7 +192,8 @@ def run_gpu(args, wl, world, rank, local):
     max_ctx = prompt + max(wl.decode_steps, total_steps)
     scale = 1.0 / np.sqrt(d)
 
-    pol = hwkv.make_policy(L, Hkv, Hq, d, B, max_ctx, wl.windows)
+    pol = hwkv.make_policy(L, Hkv, Hq, d, B, max_ctx, wl.windows,
+                           kv_format=hwkv.HWKV_KV_FP8_E4M3 if fp8 else hwkv.HWKV_KV_BF16)
     nbytes = hwkv.hwkv_required_bytes(pol)
     arena = torch.empty(nbytes, dtype=torch.uint8, device=dev)
     cache = hwkv.hwkv_alloc(pol, arena, nbytes, s)
@@ -229,7 +236,7 @@ def run_gpu(args, wl, world, rank, local):
     # a layer-step that reads less than twice the L2 would run from L2 on repeats:
     # then every timed step is preceded by a read of a 2 x L2 buffer, outside its
     # events (a read leaves clean lines, so no write-back competes with the step)
-    flush = max(decode_bytes(wl, max_ctx, prompt + 1)) < 2 * L2_BYTES
+    flush = max(decode_bytes(wl, max_ctx, prompt + 1, fp8)) < 2 * L2_BYTES
     scrub = torch.ones(2 * L2_BYTES // 4, dtype=torch.float32, device=dev) if flush else None
     scrub_out = torch.empty((), dtype=torch.float32, device=dev) if flush else None
     step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -275,7 +282,7 @@ def run_gpu(args, wl, world, rank, local):
     dec_ms, app_ms, dec_bytes, step_bytes = [], [], [], []
     for j in range(args.steps):
         t = t_first + j + 1
-        per_layer = decode_bytes(wl, max_ctx, t)
+        per_layer = decode_bytes(wl, max_ctx, t, fp8)
         e0, e1, e2 = ev[j]
         app_ms.append(e0.elapsed_time(e1))
         dec_ms.append(e1.elapsed_time(e2))
@@ -379,6 +386,7 @@ def run_gpu(args, wl, world, rank, local):
                 achieved_gbs=achieved_gbs, step_bytes=step_bytes, clocks=clocks,
                 t_first=t_first, t_end=t_end, resid_bytes=resid_bytes,
                 launches=args.steps * L * 2, e2e_steps=e2e_steps, max_ctx=max_ctx, flush=flush,
+                steps=args.steps,
                 graph_value=graph_value, graph_ms=graph_ms, graph_steps=graph_steps)
 
 
@@ -615,6 +623,10 @@ def main():
                              "budget161k_r75", "budget161k_r100"])
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=32)
+    ap.add_argument("--kv", choices=["bf16", "fp8"], default="bf16",
+                    help="cache format of the timed decode (fp8: E4M3 codes + row scales)")
+    ap.add_argument("--no-fp8", action="store_true",
+                    help="skip the secondary 8-bit-cache decode measurement")
     ap.add_argument("--prefill-reps", type=int, default=3)
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -647,7 +659,7 @@ def main():
               "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
               "context": wl.max_ctx, "window_levels": wl.levels, "note": wl.note,
               "parallelism": "replicas" if args.gpus > 1 else "single",
-              "l2": "inputs larger than L2"}
+              "l2": "inputs larger than L2", "kv_format": args.kv}
 
     if args.impl == "reference":
         if rank != 0:
@@ -683,7 +695,12 @@ def main():
               "config": {"workload": "prefill64k"}, "ms": pre["ms"], "flops": pre["flops"],
               "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst, "peak_source": peak_src})
         return
-    r = run_gpu(args, wl, world, rank, local)
+    r = run_gpu(args, wl, world, rank, local, fp8=args.kv == "fp8")
+    r8 = None  # the same decode with the 8-bit cache format, as a secondary line
+    if args.kv == "bf16" and not args.no_fp8 and wl.head_dim in (128, 256):
+        a8 = argparse.Namespace(**vars(args))
+        a8.steps, a8.e2e_steps = min(args.steps, 32), 2
+        r8 = run_gpu(a8, wl, world, rank, local, fp8=True)
     pre = None
     if not args.no_prefill and rank == 0:
         pre = run_prefill(args, local)
@@ -691,7 +708,7 @@ def main():
     if rank == 0 and not args.no_calib:
         cal = run_calib(local)
     cb = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.kv == "bf16":
         cb = cpu_baseline(wl, r["max_ctx"], r["t_first"] + 1)
     if rank != 0:
         return
@@ -702,7 +719,8 @@ def main():
     line = {
         "metric": metric, "value": r["value"], "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["ms"] / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "fp8-e4m3 KV, f16 mma" if args.kv == "fp8" else "bf16",
         "data": "synthetic", "config": config,
         "hbm_gbs": r["step_bytes"] / (r["ms"] / args.steps * 1e-3) / 1e9,
         "roofline": {"bound": "hbm",
@@ -727,6 +745,13 @@ def main():
                                "calls (lengths and tile plan on the device), replayed"
                                % wl.n_layers},
     }
+    if r8 is not None:
+        line["fp8_kv"] = {
+            "value": r8["value"], "unit": "tokens/s", "ms_per_step": r8["ms"] / r8["steps"],
+            "steps": r8["steps"], "decode_gbs": r8["achieved_gbs"], "frac": r8["achieved_gbs"] / hbm,
+            "bytes_per_launch": r8["bytes_avg"], "graph_value": r8["graph_value"],
+            "note": "same workload with the cache in E4M3 codes + one fp32 scale per row; "
+                    "bytes counted as stored (codes and scales)"}
     if pre is not None:
         line["prefill"] = {"workload": "prefill64k", "tflops": pre["tflops"],
                            "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst,

@@ -58,6 +58,22 @@ typedef enum {
 #define HWKV_WINDOW_FULL 0
 
 /*
+ * Cache format p_KV (Sec. 3.1: the nominal storage of Eq. nominal-storage is
+ * per format, through the effective precisions b^K, b^V).
+ *   HWKV_KV_BF16:     K and V rows in bf16 (b^K = b^V = 2 bytes).
+ *   HWKV_KV_FP8_E4M3: K and V rows as 8-bit E4M3 codes (1 sign, 4 exponent bits
+ *     with bias 7, 3 mantissa bits, largest finite 448) with one fp32 scale per
+ *     stored row (one token of one KV head): s = amax / 448, code = nearest E4M3
+ *     value of x / s (ties to even, saturating), value = code * s; a zero row
+ *     stores s = 0. Effective precision (d + 4) / d bytes per element. Attention
+ *     reads the dequantised rows (the paper: when the format changes execution,
+ *     every compared output uses it). head_dim 128 or 256; hwkv_prefill is not
+ *     built for it (rows enter through hwkv_append / the decode steps).
+ */
+#define HWKV_KV_BF16 0
+#define HWKV_KV_FP8_E4M3 1
+
+/*
  * The policy matrix a (Sec. 3.1, Eq. for a_{lh}; App. "Runtime Realization":
  * a static layer x KV-head matrix loaded once).
  *   windows[l * n_kv_heads + h] = W_{lh} in tokens (> 0), or HWKV_WINDOW_FULL.
@@ -72,7 +88,7 @@ typedef struct {
   int32_t n_q_heads;
   int32_t head_dim;
   int32_t batch;
-  int32_t reserved;
+  int32_t kv_format; /* HWKV_KV_BF16 or HWKV_KV_FP8_E4M3 */
   int64_t max_ctx;
   const int64_t* windows;
 } hwkv_policy;
@@ -340,8 +356,9 @@ HWKV_API hwkv_status hwkv_policy_load(const char* path, char* artifact, size_t a
                                       int64_t* windows_out, size_t capacity);
 
 /*
- * Resident K+V bytes (Sec. 3.1, Eq. nominal-storage with C = t, bf16 K and V,
- * per row): sum over KV heads and rows b of min(cap, t_b) * head_dim * 2 * 2
+ * Resident K+V bytes (Sec. 3.1, Eq. nominal-storage with C = t, per row): sum
+ * over KV heads and rows b of min(cap, t_b) * (head_dim * 2 * 2) for bf16, or
+ * min(cap, t_b) * (head_dim + 4) * 2 for the 8-bit format (codes and scales)
  * (idle rows hold nothing), for one layer, or summed over all layers when
  * layer == -1. Host-only.
  */
@@ -360,11 +377,17 @@ HWKV_API hwkv_status hwkv_ring_capacity(const hwkv_cache* cache, int32_t layer, 
 
 /*
  * Copies the ring of (layer, batch row b, kv_head) to host buffers
- * k_host, v_host of cap * head_dim bf16 each (slot-major). Synchronizes the
- * device. For tests and debugging.
+ * k_host, v_host of cap * head_dim elements each (slot-major): bf16, or E4M3
+ * codes (1 byte) for HWKV_KV_FP8_E4M3. Synchronizes the device. For tests and
+ * debugging.
  */
 HWKV_API hwkv_status hwkv_debug_copy_ring(const hwkv_cache* cache, int32_t layer, int32_t b,
                                  int32_t kv_head, void* k_host, void* v_host);
+
+/* HWKV_KV_FP8_E4M3 only: the cap fp32 row scales of that ring's K and V
+ * (slot-major), as hwkv_debug_copy_ring. */
+HWKV_API hwkv_status hwkv_debug_copy_scales(const hwkv_cache* cache, int32_t layer, int32_t b,
+                                            int32_t kv_head, float* k_scales, float* v_scales);
 
 /*
  * Synchronizes the device and reads the cache's kernel error word; returns

@@ -20,6 +20,7 @@ HEADER = os.path.join(os.path.dirname(_HERE), "include", "hwkv.h")
 HWKV_OK, HWKV_EINVAL, HWKV_ENOMEM, HWKV_ECAPACITY = 0, 1, 2, 3
 HWKV_ECUDA, HWKV_EKERNEL, HWKV_EUNSUPPORTED = 4, 5, 6
 HWKV_WINDOW_FULL = 0
+HWKV_KV_BF16, HWKV_KV_FP8_E4M3 = 0, 1
 STATUS_NAMES = {0: "HWKV_OK", 1: "HWKV_EINVAL", 2: "HWKV_ENOMEM", 3: "HWKV_ECAPACITY",
                 4: "HWKV_ECUDA", 5: "HWKV_EKERNEL", 6: "HWKV_EUNSUPPORTED"}
 
@@ -33,15 +34,16 @@ class HwkvError(RuntimeError):
 class hwkv_policy(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
                 ("n_q_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
-                ("batch", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("batch", ctypes.c_int32), ("kv_format", ctypes.c_int32),
                 ("max_ctx", ctypes.c_int64), ("windows", ctypes.POINTER(ctypes.c_int64))]
 
 
-def make_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, max_ctx, windows):
+def make_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, max_ctx, windows,
+                kv_format=HWKV_KV_BF16):
     """hwkv_policy with its windows array ([n_layers * n_kv_heads] int64, 0 = full)
     kept alive on the returned object."""
     w = np.ascontiguousarray(np.asarray(windows, dtype=np.int64).ravel())
-    pol = hwkv_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, 0, max_ctx,
+    pol = hwkv_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, kv_format, max_ctx,
                       w.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)))
     pol._windows_keepalive = w
     return pol
@@ -100,6 +102,7 @@ def lib():
             "hwkv_seq_len": [_vp, _i32, ctypes.POINTER(_i64)],
             "hwkv_ring_capacity": [_vp, _i32, _i32, ctypes.POINTER(_i64)],
             "hwkv_debug_copy_ring": [_vp, _i32, _i32, _i32, _vp, _vp],
+            "hwkv_debug_copy_scales": [_vp, _i32, _i32, _i32, _vp, _vp],
             "hwkv_sync_check": [_vp],
             "hwkv_calib_workspace_bytes": [ctypes.POINTER(hwkv_calib_desc),
                                            ctypes.POINTER(ctypes.c_size_t)],
@@ -254,13 +257,24 @@ def hwkv_ring_capacity(cache, layer, kv_head):
     return v.value
 
 
-def hwkv_debug_copy_ring(cache, layer, b, kv_head, head_dim):
-    """(K, V) of one ring as uint16 bf16 bit arrays [cap, head_dim]."""
+def hwkv_debug_copy_ring(cache, layer, b, kv_head, head_dim, kv_format=HWKV_KV_BF16):
+    """(K, V) of one ring, [cap, head_dim]: uint16 bf16 bits, or uint8 E4M3 codes."""
     cap = hwkv_ring_capacity(cache, layer, kv_head)
-    k = np.zeros((cap, head_dim), dtype=np.uint16)
-    v = np.zeros((cap, head_dim), dtype=np.uint16)
+    dt = np.uint8 if kv_format == HWKV_KV_FP8_E4M3 else np.uint16
+    k = np.zeros((cap, head_dim), dtype=dt)
+    v = np.zeros((cap, head_dim), dtype=dt)
     _check(lib().hwkv_debug_copy_ring(cache, layer, b, kv_head,
                                       k.ctypes.data_as(_vp), v.ctypes.data_as(_vp)))
+    return k, v
+
+
+def hwkv_debug_copy_scales(cache, layer, b, kv_head):
+    """(K scales, V scales) of one 8-bit ring, float32 [cap]."""
+    cap = hwkv_ring_capacity(cache, layer, kv_head)
+    k = np.zeros(cap, dtype=np.float32)
+    v = np.zeros(cap, dtype=np.float32)
+    _check(lib().hwkv_debug_copy_scales(cache, layer, b, kv_head, k.ctypes.data_as(_vp),
+                                        v.ctypes.data_as(_vp)))
     return k, v
 
 

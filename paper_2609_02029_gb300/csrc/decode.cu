@@ -243,8 +243,8 @@ struct TileWalker {
     const int64_t len = min((int64_t)n - start, rem);
     ti.start = start;
     ti.len = (int)len;
-    ti.k_row = du.k_row0 + (int64_t)ti.b * du.cap + start;
-    ti.v_row = du.v_row0 + (int64_t)ti.b * du.cap + start;
+    ti.k_row = du.k_row0 + (int64_t)ti.b * du.stride + start;
+    ti.v_row = du.v_row0 + (int64_t)ti.b * du.stride + start;
     ti.s_new = (int64_t)len_b % du.cap;
     ti.single = start == 0 && len == n;
     ti.tile = 2 * (int)blockIdx.x + (first ? 0 : 1);
@@ -277,32 +277,41 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
-template <int D>
+// FP8: K/V stages hold E4M3 codes (one byte per channel, 128 channels per
+// 128-byte slab) and each stage's 64 K and 64 V row scales arrive beside it; every
+// consumer warp dequantises its 16 V rows into a private f16 scratch.
+template <int D, bool FP8>
 struct DecodeCfg {
-  static constexpr int kSlabs = D / 64;
+  static constexpr int kChanPerSlab = FP8 ? 128 : 64;
+  static constexpr int kSlabs = D / kChanPerSlab;
   static constexpr int kTileBytes = kSlabs * kSlabBytes;  // 64 tokens of K (or V)
   static constexpr int kStageBytes = 2 * kTileBytes;
-  static constexpr int kStages = D == 256 ? 3 : (D == 128 ? 6 : 8);
+  static constexpr int kStages = FP8 ? (D == 256 ? 4 : 8) : (D == 256 ? 3 : (D == 128 ? 6 : 8));
+  static constexpr int kScaleBytes = FP8 ? kStages * 2 * kStageTokens * 4 : 0;
+  static constexpr int kScratchBytes = FP8 ? kDecodeWarps * 16 * D * 2 : 0;  // f16 V rows
   static constexpr int kRedLd = D + 4;  // padded row of the cross-warp merge area (floats)
   static constexpr int kRedBytes = kDecodeWarps * kMaxGroup * kRedLd * 4;
   static constexpr int kMlBytes = kDecodeWarps * kMaxGroup * 8;
-  static constexpr int kSmem = kStages * kStageBytes + kRedBytes + kMlBytes + 2 * kStages * 8 + 1024;
+  static constexpr int kSmem = kStages * kStageBytes + kScratchBytes + kScaleBytes + kRedBytes +
+                               kMlBytes + 2 * kStages * 8 + 1024;
 };
 
 }  // namespace
 
-template <int D>
+template <int D, bool FP8>
 __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     decode_split_kernel(const __grid_constant__ CUtensorMap k_map,
                         const __grid_constant__ CUtensorMap v_map, const DecodeParams p) {
-  using C = DecodeCfg<D>;
+  using C = DecodeCfg<D, FP8>;
   constexpr int STAGES = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  float* red_o = reinterpret_cast<float*>(smem + STAGES * C::kStageBytes);
-  float2* red_ml = reinterpret_cast<float2*>(smem + STAGES * C::kStageBytes + C::kRedBytes);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::kStageBytes + C::kRedBytes +
-                                               C::kMlBytes);
+  uint8_t* scratch = smem + STAGES * C::kStageBytes;               // FP8: [warp][16 rows] f16
+  float* stage_scales = reinterpret_cast<float*>(scratch + C::kScratchBytes);  // [stage][K|V][64]
+  uint8_t* tail = scratch + C::kScratchBytes + C::kScaleBytes;
+  float* red_o = reinterpret_cast<float*>(tail);
+  float2* red_ml = reinterpret_cast<float2*>(tail + C::kRedBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(tail + C::kRedBytes + C::kMlBytes);
   uint64_t* empty = full + STAGES;
 
   const int warp = threadIdx.x >> 5;
@@ -343,15 +352,20 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
         }
         uint8_t* kdst = smem + s * C::kStageBytes;
         uint8_t* vdst = kdst + C::kTileBytes;
-        mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+        mbar_arrive_expect_tx(&full[s], C::kStageBytes + (FP8 ? 2 * kStageTokens * 4 : 0));
         const int32_t krow = (int32_t)(ti.k_row + (int64_t)st * kStageTokens);
         const int32_t vrow = (int32_t)(ti.v_row + (int64_t)st * kStageTokens);
 #pragma unroll
         for (int sl = 0; sl < C::kSlabs; ++sl)
-          tma_load_2d(kdst + sl * kSlabBytes, &k_map, sl * 64, krow, &full[s]);
+          tma_load_2d(kdst + sl * kSlabBytes, &k_map, sl * C::kChanPerSlab, krow, &full[s]);
 #pragma unroll
         for (int sl = 0; sl < C::kSlabs; ++sl)
-          tma_load_2d(vdst + sl * kSlabBytes, &v_map, sl * 64, vrow, &full[s]);
+          tma_load_2d(vdst + sl * kSlabBytes, &v_map, sl * C::kChanPerSlab, vrow, &full[s]);
+        if constexpr (FP8) {  // rows are 64-aligned, so each 256-byte scale run is too
+          float* sdst = stage_scales + s * 2 * kStageTokens;
+          bulk_load(sdst, p.scales + krow, kStageTokens * 4, &full[s]);
+          bulk_load(sdst + kStageTokens, p.scales + vrow, kStageTokens * 4, &full[s]);
+        }
       }
     }
     if (!ok) {
@@ -380,16 +394,34 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
   while (wk.next(p, ti)) {
     const int n_st = (ti.len + kStageTokens - 1) / kStageTokens;
 
-    // Q^T as mma B fragments: b0 = channels 16kk + qk + {0,1}, b1 = +8; column = head qn
+    // Q^T as mma B fragments, column = head qn. bf16: b0 = channels 16kk + qk +
+    // {0,1}, b1 = +8. FP8 (f16 mma): the E4M3 A fragments of 32 channels arrive as
+    // 4 consecutive channels per lane, so mma m of step kk contracts over channels
+    // 32kk + 4(lane&3) + 2m + {0,1} (b0) and the same + 16 (b1); Q follows that order
     uint32_t qf[D / 16][2];
     {
       const bool qv = qn < p.group;
       const __nv_bfloat16* qrow =
           p.q + ((int64_t)ti.b * p.n_q_heads + (int64_t)ti.h * p.group + (qv ? qn : 0)) * D;
+      if constexpr (!FP8) {
 #pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {
-        qf[kk][0] = qv ? *reinterpret_cast<const uint32_t*>(qrow + kk * 16 + qk) : 0u;
-        qf[kk][1] = qv ? *reinterpret_cast<const uint32_t*>(qrow + kk * 16 + 8 + qk) : 0u;
+        for (int kk = 0; kk < D / 16; ++kk) {
+          qf[kk][0] = qv ? *reinterpret_cast<const uint32_t*>(qrow + kk * 16 + qk) : 0u;
+          qf[kk][1] = qv ? *reinterpret_cast<const uint32_t*>(qrow + kk * 16 + 8 + qk) : 0u;
+        }
+      } else {
+        auto f16pair = [&](int ch) -> uint32_t {
+          const uint32_t x = *reinterpret_cast<const uint32_t*>(qrow + ch);
+          return pack_f16(__uint_as_float(x << 16), __uint_as_float(x & 0xffff0000u));
+        };
+#pragma unroll
+        for (int kk = 0; kk < D / 32; ++kk)
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            const int ch = kk * 32 + (lane & 3) * 4 + 2 * m;
+            qf[2 * kk + m][0] = qv ? f16pair(ch) : 0u;
+            qf[2 * kk + m][1] = qv ? f16pair(ch + 16) : 0u;
+          }
       }
     }
 
@@ -409,11 +441,71 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
       }
       const uint32_t kbase = smem_u32(smem + s * C::kStageBytes);
       const uint32_t vbase = kbase + C::kTileBytes;
+      float* ksc = stage_scales + s * 2 * kStageTokens;  // FP8: this stage's row scales
+      float* vsc = ksc + kStageTokens;
       if (p.k_new != nullptr) {
         // fused step: the new token's slot may lie in this stage; the warp owning that
         // row replaces the staged (stale) row with the new K/V and writes the ring row
         const int64_t row_in = ti.s_new - (ti.start + (int64_t)st * kStageTokens);
-        if (row_in >= w * 16 && row_in < w * 16 + 16) {
+        if constexpr (FP8) {
+         if (row_in >= w * 16 && row_in < w * 16 + 16) {
+          // quantise as the append does: amax over the row, s = amax / 448, codes of x / s
+          constexpr int PER = D / 32;
+          const int r = (int)row_in;
+#pragma unroll
+          for (int kv = 0; kv < 2; ++kv) {
+            const __nv_bfloat16* src =
+                (kv ? p.v_new : p.k_new) + ((int64_t)ti.b * p.n_units + ti.h) * D + lane * PER;
+            uint32_t raw[PER / 2];
+            if constexpr (PER == 8) {
+              const uint4 v = *reinterpret_cast<const uint4*>(src);
+              raw[0] = v.x; raw[1] = v.y; raw[2] = v.z; raw[3] = v.w;
+            } else {
+              const uint2 v = *reinterpret_cast<const uint2*>(src);
+              raw[0] = v.x; raw[1] = v.y;
+            }
+            float x[PER], amax = 0.f;
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+              x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
+              amax = fmaxf(amax, fabsf(x[j]));
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1)
+              amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+            const float sc = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
+            uint32_t cw[PER / 4];
+#pragma unroll
+            for (int j = 0; j < PER; j += 4) {
+              uint32_t c01 = 0, c23 = 0;
+              if (amax > 0.f) {
+                c01 = f32x2_to_e4m3x2(__fdiv_rn(x[j], sc), __fdiv_rn(x[j + 1], sc));
+                c23 = f32x2_to_e4m3x2(__fdiv_rn(x[j + 2], sc), __fdiv_rn(x[j + 3], sc));
+              }
+              cw[j / 4] = c01 | (c23 << 16);
+            }
+            const int64_t ring = (kv ? ti.v_row : ti.k_row) - ti.start + ti.s_new;
+            uint8_t* g = reinterpret_cast<uint8_t*>(p.arena) + ring * D + lane * PER;
+            const int c0 = lane * PER;  // first channel of this lane
+            const uint32_t a = (kv ? vbase : kbase) + (c0 >> 7) * kSlabBytes +
+                               swz128(r, (c0 & 127) >> 4) + (c0 & 15);
+            if constexpr (PER == 8) {
+              *reinterpret_cast<uint2*>(g) = make_uint2(cw[0], cw[1]);
+              asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(a), "r"(cw[0]), "r"(cw[1])
+                           : "memory");
+            } else {
+              *reinterpret_cast<uint32_t*>(g) = cw[0];
+              asm volatile("st.shared.b32 [%0], %1;" ::"r"(a), "r"(cw[0]) : "memory");
+            }
+            if (lane == 0) {
+              p.scales[ring] = sc;
+              (kv ? vsc : ksc)[r] = sc;
+            }
+          }
+          fence_proxy_async_smem();  // these generic writes precede the next copy into the stage
+          __syncwarp();
+         }
+        } else if (row_in >= w * 16 && row_in < w * 16 + 16) {
           const int r = (int)row_in;
           const __nv_bfloat16* src_k = p.k_new + ((int64_t)ti.b * p.n_units + ti.h) * D;
           const __nv_bfloat16* src_v = p.v_new + ((int64_t)ti.b * p.n_units + ti.h) * D;
@@ -439,18 +531,75 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
       {
         const int r = w * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
         const int csel = lane >> 4;
+        if constexpr (!FP8) {
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          uint32_t a0, a1, a2, a3;
-          ldsm_x4(kbase + (kk >> 2) * kSlabBytes + swz128(r, (kk & 3) * 2 + csel), a0, a1, a2,
-                  a3);
-          if (kk & 1)
-            mma_bf16_16816(sb, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
-          else
-            mma_bf16_16816(sa, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+          for (int kk = 0; kk < D / 16; ++kk) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4(kbase + (kk >> 2) * kSlabBytes + swz128(r, (kk & 3) * 2 + csel), a0, a1, a2,
+                    a3);
+            if (kk & 1)
+              mma_bf16_16816(sb, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+            else
+              mma_bf16_16816(sa, a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+          }
+        } else {
+          // 32 channels per step: the x4 load gives every lane 4 consecutive E4M3
+          // channels of two rows, split into the two f16 mmas of Q's channel order
+#pragma unroll
+          for (int kk = 0; kk < D / 32; ++kk) {
+            uint32_t a0, a1, a2, a3, l0, l1, l2, l3, h0, h1, h2, h3;
+            ldsm_x4(kbase + (kk >> 2) * kSlabBytes + swz128(r, (kk & 3) * 2 + csel), a0, a1, a2,
+                    a3);
+            e4m3x4_to_f16x2(a0, l0, h0);
+            e4m3x4_to_f16x2(a1, l1, h1);
+            e4m3x4_to_f16x2(a2, l2, h2);
+            e4m3x4_to_f16x2(a3, l3, h3);
+            mma_f16_16816(sa, l0, l1, l2, l3, qf[2 * kk][0], qf[2 * kk][1]);
+            mma_f16_16816(sb, h0, h1, h2, h3, qf[2 * kk + 1][0], qf[2 * kk + 1][1]);
+          }
         }
       }
       float s0 = sa[0] + sb[0], s1 = sa[1] + sb[1], s2 = sa[2] + sb[2], s3 = sa[3] + sb[3];
+      float vsA = 1.f, vsB = 1.f;  // FP8: V row scales of this lane's two tokens
+      if constexpr (FP8) {
+        const int tA = w * 16 + (lane >> 2);
+        const float ksA = ksc[tA], ksB = ksc[tA + 8];
+        vsA = vsc[tA];
+        vsB = vsc[tA + 8];
+        s0 *= ksA;
+        s1 *= ksA;
+        s2 *= ksB;
+        s3 *= ksB;
+        // dequantise this warp's 16 V rows into its f16 scratch (same swizzled layout
+        // as a bf16 V tile), then the stage can be refilled
+        const int rr = lane >> 1, hf = lane & 1;
+        const uint32_t sw = smem_u32(scratch) + w * (16 * D * 2);
+        constexpr int CH = D / 32;  // 16-byte E4M3 chunks per lane
+#pragma unroll
+        for (int j = 0; j < CH; ++j) {
+          const int g = hf * CH + j;  // channels 16g .. 16g + 15
+          uint32_t x0, x1, x2, x3;
+          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                       : "=r"(x0), "=r"(x1), "=r"(x2), "=r"(x3)
+                       : "r"(vbase + (g >> 3) * kSlabBytes + swz128(w * 16 + rr, g & 7))
+                       : "memory");
+          uint32_t f[8];
+          e4m3x4_to_f16x2(x0, f[0], f[1]);
+          e4m3x4_to_f16x2(x1, f[2], f[3]);
+          e4m3x4_to_f16x2(x2, f[4], f[5]);
+          e4m3x4_to_f16x2(x3, f[6], f[7]);
+          const uint32_t d0 = sw + (g >> 2) * (16 * 128) + swz128(rr, (g & 3) * 2);
+          const uint32_t d1 = sw + (g >> 2) * (16 * 128) + swz128(rr, (g & 3) * 2 + 1);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(d0), "r"(f[0]), "r"(f[1]),
+                       "r"(f[2]), "r"(f[3])
+                       : "memory");
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(d1), "r"(f[4]), "r"(f[5]),
+                       "r"(f[6]), "r"(f[7])
+                       : "memory");
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[s]);
+      }
       const int tok = st * kStageTokens + w * 16 + (lane >> 2);
       if (tok >= ti.len) s0 = s1 = -INFINITY;
       if (tok + 8 >= ti.len) s2 = s3 = -INFINITY;
@@ -481,24 +630,35 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
           o[mt][3] *= alB;
         }
       }
-      const uint32_t pb0 = movmatrix_trans(pack_bf16(p0, p1));
-      const uint32_t pb1 = movmatrix_trans(pack_bf16(p2, p3));
-
-      // O^T += V^T . P^T
+      // O^T += V^T . P^T  (FP8: the V row scales ride on P; the sums l do not)
+      const uint32_t pb0 = movmatrix_trans(FP8 ? pack_f16(p0 * vsA, p1 * vsA) : pack_bf16(p0, p1));
+      const uint32_t pb1 = movmatrix_trans(FP8 ? pack_f16(p2 * vsB, p3 * vsB) : pack_bf16(p2, p3));
       {
         const int mi = lane >> 3;
-        const int r = w * 16 + (lane & 7) + (mi >> 1) * 8;
         const int csel = mi & 1;
+        if constexpr (!FP8) {
+          const int r = w * 16 + (lane & 7) + (mi >> 1) * 8;
 #pragma unroll
-        for (int mt = 0; mt < D / 16; ++mt) {
-          uint32_t a0, a1, a2, a3;
-          ldsm_x4_t(vbase + (mt >> 2) * kSlabBytes + swz128(r, (mt & 3) * 2 + csel), a0, a1, a2,
-                    a3);
-          mma_bf16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+          for (int mt = 0; mt < D / 16; ++mt) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4_t(vbase + (mt >> 2) * kSlabBytes + swz128(r, (mt & 3) * 2 + csel), a0, a1,
+                      a2, a3);
+            mma_bf16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+          }
+        } else {
+          const int rl = (lane & 7) + (mi >> 1) * 8;
+          const uint32_t sw = smem_u32(scratch) + w * (16 * D * 2);
+#pragma unroll
+          for (int mt = 0; mt < D / 16; ++mt) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4_t(sw + (mt >> 2) * (16 * 128) + swz128(rl, (mt & 3) * 2 + csel), a0, a1, a2,
+                      a3);
+            mma_f16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+          }
         }
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[s]);
+      if (!FP8 && lane == 0) mbar_arrive(&empty[s]);
     }
 
     // ---- merge the four warps' partials of this tile in shared memory
@@ -647,11 +807,17 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
 
 int decode_smem_bytes(int head_dim) {
   switch (head_dim) {
-    case 64: return DecodeCfg<64>::kSmem;
-    case 128: return DecodeCfg<128>::kSmem;
-    case 256: return DecodeCfg<256>::kSmem;
+    case 64: return DecodeCfg<64, false>::kSmem;
+    case 128: return DecodeCfg<128, false>::kSmem;
+    case 256: return DecodeCfg<256, false>::kSmem;
     default: return -1;
   }
+}
+
+template <int D, bool FP8>
+static cudaError_t opt_in() {
+  return cudaFuncSetAttribute(decode_split_kernel<D, FP8>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeCfg<D, FP8>::kSmem);
 }
 
 // The shared-memory opt-in of the split kernels, once per device (host calls
@@ -666,33 +832,37 @@ cudaError_t decode_prepare_device() {
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(mu);
   if (done[dev]) return cudaSuccess;
-  e = cudaFuncSetAttribute(decode_split_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           DecodeCfg<64>::kSmem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(decode_split_kernel<128>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeCfg<128>::kSmem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(decode_split_kernel<256>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeCfg<256>::kSmem);
+  e = opt_in<64, false>();
+  if (e == cudaSuccess) e = opt_in<128, false>();
+  if (e == cudaSuccess) e = opt_in<256, false>();
+  if (e == cudaSuccess) e = opt_in<128, true>();
+  if (e == cudaSuccess) e = opt_in<256, true>();
   if (e == cudaSuccess) done[dev] = true;
   return e;
 }
 
-template <int D>
+template <int D, bool FP8>
 static cudaError_t launch_decode_t(const DecodeParams& p, const CUtensorMap& kmap,
                                    const CUtensorMap& vmap, int grid, cudaStream_t s) {
   cudaError_t e = decode_prepare_device();
   if (e != cudaSuccess) return e;
-  return launch_pdl(decode_split_kernel<D>, dim3(grid), dim3((kDecodeWarps + 1) * 32),
-                    DecodeCfg<D>::kSmem, s, kmap, vmap, p);
+  return launch_pdl(decode_split_kernel<D, FP8>, dim3(grid), dim3((kDecodeWarps + 1) * 32),
+                    DecodeCfg<D, FP8>::kSmem, s, kmap, vmap, p);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& kmap, const CUtensorMap& vmap,
-                          int head_dim, int grid, cudaStream_t s) {
+                          int head_dim, int grid, cudaStream_t s, bool fp8) {
+  if (fp8) {
+    switch (head_dim) {
+      case 128: return launch_decode_t<128, true>(p, kmap, vmap, grid, s);
+      case 256: return launch_decode_t<256, true>(p, kmap, vmap, grid, s);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (head_dim) {
-    case 64: return launch_decode_t<64>(p, kmap, vmap, grid, s);
-    case 128: return launch_decode_t<128>(p, kmap, vmap, grid, s);
-    case 256: return launch_decode_t<256>(p, kmap, vmap, grid, s);
+    case 64: return launch_decode_t<64, false>(p, kmap, vmap, grid, s);
+    case 128: return launch_decode_t<128, false>(p, kmap, vmap, grid, s);
+    case 256: return launch_decode_t<256, false>(p, kmap, vmap, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -32,7 +32,8 @@ constexpr int kDecodeSlots = 512;  // decode partial slots in the cache workspac
 struct DecodeUnit {
   int64_t k_row0;   // arena row of (this KV head, batch row 0) in the K region
   int64_t v_row0;   // same in the V region
-  int64_t cap;      // ring capacity; batch row b starts at row0 + b * cap
+  int64_t cap;      // ring capacity (slots)
+  int64_t stride;   // rows between batch rows: batch row b starts at row0 + b * stride
 };
 
 // a tile of explicit key rows (SeqCalib replay): rows k_row.. / v_row.. of the trace
@@ -60,7 +61,8 @@ struct DecodeParams {
   // the new token's row is patched into the staged tile and written to the ring
   const __nv_bfloat16* k_new;  // null: plain decode over the current ring contents
   const __nv_bfloat16* v_new;
-  __nv_bfloat16* arena;        // K/V rows: row r at arena + r * D
+  __nv_bfloat16* arena;        // K/V rows: row r at arena + r * D (bytes r * D for 8-bit)
+  float* scales;               // 8-bit format: fp32 scale of K/V row r at scales[r]
   const CalibTile* tiles;      // table mode: tiles[n_tiles]; every tile leaves a partial
   // ring mode: per-row lengths of this layer on the device, [batch]: tokens held by
   // row b before this call, -1 = idle row. With lens_inc = 1 (fused step) the new
@@ -86,7 +88,7 @@ struct CalibCombineParams {
 
 // ------------------------------------------------------------------ append
 struct AppendUnit {
-  int64_t k_row0, v_row0, cap;
+  int64_t k_row0, v_row0, cap, stride;
 };
 
 struct AppendParams {
@@ -98,8 +100,9 @@ struct AppendParams {
   int64_t d;       // head_dim
   const __nv_bfloat16* k;  // [batch][n][n_units][d]
   const __nv_bfloat16* v;
-  __nv_bfloat16* k_arena;  // row r at k_arena + r * d
+  __nv_bfloat16* k_arena;  // row r at k_arena + r * d (bytes r * d for 8-bit)
   __nv_bfloat16* v_arena;
+  float* scales;           // 8-bit format: scale of row r at scales[r]
   AppendUnit u[kMaxKvHeads];
 };
 
@@ -107,6 +110,7 @@ struct AppendParams {
 struct PrefillUnit {
   int64_t k_row0, v_row0, cap;
   int64_t window;  // 0 = full
+  int64_t stride;  // rows between batch rows
 };
 
 struct PrefillParams {
@@ -126,9 +130,10 @@ struct PrefillParams {
 };
 
 // launchers (defined in the kernel translation units); return cudaGetLastError()
-cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& k_map,
-                          const CUtensorMap& v_map, int head_dim, int grid, cudaStream_t s);
+                          const CUtensorMap& v_map, int head_dim, int grid, cudaStream_t s,
+                          bool fp8 = false);
 cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cudaStream_t s);
 cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s);
 cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtensorMap& q_map,
@@ -259,6 +264,16 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
+// plain bulk copy global -> shared (both 16-byte aligned, bytes a multiple of 16)
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes),
+      "r"(smem_u32(bar))
+      : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -298,6 +313,39 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
       "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
+                                              uint32_t a2, uint32_t a3, uint32_t b0,
+                                              uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// four E4M3 codes (bytes 0..3 of x) -> f16 pairs: lo = bytes 0, 1; hi = bytes 2, 3
+__device__ __forceinline__ void e4m3x4_to_f16x2(uint32_t x, uint32_t& lo, uint32_t& hi) {
+  asm("{\n\t.reg .b16 l, h;\n\t"
+      "mov.b32 {l, h}, %2;\n\t"
+      "cvt.rn.f16x2.e4m3x2 %0, l;\n\t"
+      "cvt.rn.f16x2.e4m3x2 %1, h;\n\t}"
+      : "=r"(lo), "=r"(hi)
+      : "r"(x));
+}
+
+// two floats -> two E4M3 codes (round to nearest even, saturating): byte 0 = lo
+__device__ __forceinline__ uint32_t f32x2_to_e4m3x2(float lo, float hi) {
+  uint16_t d;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
 }
 
 __device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a) {

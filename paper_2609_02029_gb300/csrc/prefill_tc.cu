@@ -235,8 +235,8 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
 #pragma unroll
       for (int sl = 0; sl < C::kSlabs; ++sl)
         tma_load_3d(sQ + sl * C::kQSlab, &q_map, sl * 64, h * G, qrow, q_full);
-      const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.cap;
-      const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.cap;
+      const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;
+      const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.stride;
       uint32_t it = 0;
       int hist;
       int64_t j0;

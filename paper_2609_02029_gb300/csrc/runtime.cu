@@ -49,6 +49,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 struct Unit {
   int64_t window;  // effective: 0 = full
   int64_t cap;
+  int64_t stride;  // rows per batch row: cap, rounded up to 64 in the 8-bit format
   int64_t k_row0, v_row0;
 };
 
@@ -56,6 +57,7 @@ struct Layout {
   std::vector<Unit> units;  // [layer * n_kv_heads + h]
   int64_t rows = 0;         // K rows (= V rows)
   size_t ring_bytes = 0;    // K + V
+  size_t scale_off = 0;     // 8-bit format: fp32 row scales [2 * rows + 64]
   size_t part_o_off = 0, part_ml_off = 0, err_off = 0, lens_off = 0, plan_off = 0, total = 0;
   int slots = 0;  // decode partial slots: two per CTA of a split launch
 };
@@ -80,6 +82,10 @@ hwkv_status validate(const hwkv_policy* p) {
   if (p->n_kv_heads > kMaxKvHeads)
     return fail(HWKV_EUNSUPPORTED, "n_kv_heads %d > %d", p->n_kv_heads, kMaxKvHeads);
   if (p->batch > 256) return fail(HWKV_EUNSUPPORTED, "batch %d > 256", p->batch);
+  if (p->kv_format != HWKV_KV_BF16 && p->kv_format != HWKV_KV_FP8_E4M3)
+    return fail(HWKV_EINVAL, "unknown kv_format %d", p->kv_format);
+  if (p->kv_format == HWKV_KV_FP8_E4M3 && p->head_dim != 128 && p->head_dim != 256)
+    return fail(HWKV_EUNSUPPORTED, "the 8-bit format is built for head_dim 128 and 256");
   return HWKV_OK;
 }
 
@@ -92,6 +98,8 @@ Layout make_layout(const hwkv_policy* p) {
     Unit& u = L.units[i];
     u.window = (W == HWKV_WINDOW_FULL || W >= p->max_ctx) ? 0 : W;  // w >= C is full (Sec. 3.1)
     u.cap = u.window == 0 ? p->max_ctx : u.window;
+    // 8-bit rings start on 64-row boundaries: a stage's 64 scales are one aligned run
+    u.stride = p->kv_format == HWKV_KV_FP8_E4M3 ? (u.cap + 63) / 64 * 64 : u.cap;
   }
   // group by level: larger capacity first, then layer, then head
   std::vector<int> order(nu);
@@ -101,14 +109,17 @@ Layout make_layout(const hwkv_policy* p) {
   int64_t row = 0;
   for (int i : order) {
     L.units[i].k_row0 = row;
-    row += L.units[i].cap * p->batch;
+    row += L.units[i].stride * p->batch;
   }
   L.rows = row;
   for (auto& u : L.units) u.v_row0 = u.k_row0 + L.rows;
-  const size_t row_bytes = (size_t)p->head_dim * 2;
+  const bool fp8 = p->kv_format == HWKV_KV_FP8_E4M3;
+  const size_t row_bytes = (size_t)p->head_dim * (fp8 ? 1 : 2);
   L.ring_bytes = (size_t)(2 * L.rows) * row_bytes;
+  L.scale_off = align_up(L.ring_bytes, kAlign);
+  const size_t scale_bytes = fp8 ? (size_t)(2 * L.rows + kStageTokens) * 4 : 0;
   L.slots = kDecodeSlots;
-  L.part_o_off = align_up(L.ring_bytes, kAlign);
+  L.part_o_off = align_up(L.scale_off + scale_bytes, kAlign);
   L.part_ml_off = align_up(L.part_o_off + (size_t)L.slots * kMaxGroup * p->head_dim * 4, kAlign);
   L.err_off = align_up(L.part_ml_off + (size_t)L.slots * kMaxGroup * 8, kAlign);
   // per-row lengths on the device, [layer][batch] int32, then the decode plan
@@ -150,9 +161,13 @@ struct hwkv_cache {
   uint8_t* arena = nullptr;
   bool owns_arena = false;
   int num_sms = 0;
-  CUtensorMap kv_map;  // 2-D view of the K and V regions: [2 * rows][head_dim] bf16
+  CUtensorMap kv_map;  // 2-D view of the K and V regions: [2 * rows][head_dim] elements
+  bool fp8() const { return pol.kv_format == HWKV_KV_FP8_E4M3; }
+  size_t elem_bytes() const { return fp8() ? 1 : 2; }
+  // bytes one resident token of one KV head occupies (K and V, with scales)
+  size_t token_bytes() const { return fp8() ? 2 * ((size_t)pol.head_dim + 4) : 4 * (size_t)pol.head_dim; }
   __nv_bfloat16* k_base() const { return reinterpret_cast<__nv_bfloat16*>(arena); }
-  __nv_bfloat16* v_base() const { return k_base() + lay.rows * pol.head_dim; }
+  float* scales() const { return fp8() ? reinterpret_cast<float*>(arena + lay.scale_off) : nullptr; }
   float* part_o() const { return reinterpret_cast<float*>(arena + lay.part_o_off); }
   float2* part_ml() const { return reinterpret_cast<float2*>(arena + lay.part_ml_off); }
   int* err() const { return reinterpret_cast<int*>(arena + lay.err_off); }
@@ -250,11 +265,13 @@ hwkv_status hwkv_alloc(const hwkv_policy* policy, void* dev_arena, size_t arena_
     return fail(HWKV_ECUDA, "zero-fill failed: %s", cudaGetErrorString(e));
   }
   // one tensor map over both regions: rows of head_dim bf16, boxes of 64 rows x 64 channels
+  // (128-byte rows of boxes: 64 bf16 or 128 E4M3 channels)
   const cuuint64_t gdim[2] = {(cuuint64_t)c->pol.head_dim, (cuuint64_t)(2 * c->lay.rows)};
-  const cuuint64_t gstride[1] = {(cuuint64_t)c->pol.head_dim * 2};
-  const cuuint32_t box[2] = {64, (cuuint32_t)kStageTokens};
+  const cuuint64_t gstride[1] = {(cuuint64_t)c->pol.head_dim * c->elem_bytes()};
+  const cuuint32_t box[2] = {c->fp8() ? 128u : 64u, (cuuint32_t)kStageTokens};
   const cuuint32_t estride[2] = {1, 1};
-  CUresult r = encode(&c->kv_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->arena, gdim, gstride,
+  CUresult r = encode(&c->kv_map, c->fp8() ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                      2, c->arena, gdim, gstride,
                       box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
@@ -320,9 +337,10 @@ static AppendParams append_params(const hwkv_cache* c, int32_t layer, int32_t ro
   p.v = static_cast<const __nv_bfloat16*>(v);
   p.k_arena = c->k_base();
   p.v_arena = c->k_base();  // V rows are addressed by v_row0, which already includes the K region
+  p.scales = c->scales();
   for (int h = 0; h < p.n_units; ++h) {
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
-    p.u[h] = AppendUnit{u.k_row0, u.v_row0, u.cap};
+    p.u[h] = AppendUnit{u.k_row0, u.v_row0, u.cap, u.stride};
   }
   return p;
 }
@@ -350,7 +368,7 @@ hwkv_status hwkv_append_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_t
   if (!k || !v) return fail(HWKV_EINVAL, "k/v is NULL");
   if ((st = check_room(c, layer, row0, n_rows, n)) != HWKV_OK) return st;
   const AppendParams p = append_params(c, layer, row0, n_rows, k, v, n);
-  cudaError_t e = launch_append(p, static_cast<cudaStream_t>(cuda_stream));
+  cudaError_t e = launch_append(p, c->fp8(), static_cast<cudaStream_t>(cuda_stream));
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "append launch: %s", cudaGetErrorString(e));
   for (int b = row0; b < row0 + n_rows; ++b) c->row_t(layer, b) += n;
   return ok();
@@ -371,6 +389,7 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
   if (n < 0) return fail(HWKV_EINVAL, "n must be >= 0");
   if (n == 0) return ok();
   if (!q || !k || !v || !out) return fail(HWKV_EINVAL, "q/k/v/out is NULL");
+  if (c->fp8()) return fail(HWKV_EUNSUPPORTED, "prefill is not built for the 8-bit cache format");
   if ((st = check_room(c, layer, row0, n_rows, n)) != HWKV_OK) return st;
   const int64_t t_rows = c->row_t(layer, row0);
   for (int b = row0 + 1; b < row0 + n_rows; ++b)
@@ -398,7 +417,7 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
   p.err = c->err();
   for (int h = 0; h < p.n_units; ++h) {
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
-    p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window};
+    p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window, u.stride};
   }
   // tensor maps of this call's q and chunk K/V: 3-D views {d, heads, batch * n}
   auto encode = get_encode();
@@ -435,7 +454,7 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "prefill launch: %s", cudaGetErrorString(e));
   // attend first, then write the chunk's retained tokens (stream order)
   const AppendParams ap = append_params(c, layer, row0, n_rows, k, v, n);
-  e = launch_append(ap, s);
+  e = launch_append(ap, false, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "append launch: %s", cudaGetErrorString(e));
   for (int b = row0; b < row0 + n_rows; ++b) c->row_t(layer, b) += n;
   return ok();
@@ -455,7 +474,7 @@ hwkv_status hwkv_prefill(hwkv_cache* c, int32_t layer, const void* q, const void
 // step reads (an estimate is enough: it changes speed, not results).
 static int decode_grid_cap(const hwkv_cache* c, int64_t tokens) {
   const int sms = std::max(1, c->num_sms);
-  const int64_t bytes = tokens * 4 * c->pol.head_dim;
+  const int64_t bytes = tokens * (int64_t)c->token_bytes();
   constexpr int64_t kFullGridBytes = 1LL << 30;
   return (bytes >= kFullGridBytes || sms <= 16) ? sms : sms - 8;
 }
@@ -484,12 +503,13 @@ static void ring_params(const hwkv_cache* c, int32_t layer, DecodeParams& p, int
   p.lens = c->lens(layer);
   p.lens_inc = lens_inc;
   p.max_ctx = c->pol.max_ctx;
+  p.scales = c->scales();
   // a segment's fixed cost (query load, merge, partial write) ~ the time to stream
   // 256 KB of K/V at one CTA's share of HBM bandwidth, in 64-key stages
-  p.seg_cost = std::max(1, (256 << 10) / (4 * c->pol.head_dim) / kStageTokens);
+  p.seg_cost = std::max(1, (int)((256 << 10) / c->token_bytes() / kStageTokens));
   for (int h = 0; h < p.n_units; ++h) {
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
-    p.u[h] = DecodeUnit{u.k_row0, u.v_row0, u.cap};
+    p.u[h] = DecodeUnit{u.k_row0, u.v_row0, u.cap, u.stride};
   }
 }
 
@@ -531,7 +551,7 @@ static hwkv_status decode_call(hwkv_cache* c, int32_t layer, const void* q, cons
   // the host copy of the lengths sizes the grid (stale under graph capture: an estimate)
   const int grid = decode_grid_cap(c, step_tokens(c, layer, mode == kPlain ? 0 : 1));
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s);
+  cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s, c->fp8());
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
   e = launch_decode_combine(p, c->pol.head_dim, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
@@ -595,7 +615,8 @@ hwkv_status hwkv_residency_bytes(const hwkv_cache* c, int32_t layer, uint64_t* b
   if (!c || !bytes) return fail(HWKV_EINVAL, "NULL argument");
   if (layer < -1 || layer >= c->pol.n_layers) return fail(HWKV_EINVAL, "layer out of range");
   const int H = c->pol.n_kv_heads;
-  const uint64_t per_token = (uint64_t)c->pol.head_dim * 2 * 2;  // d^K b^K + d^V b^V, bf16
+  // d^K b^K + d^V b^V: bf16, or E4M3 codes plus a 4-byte scale per row
+  const uint64_t per_token = c->token_bytes();
   uint64_t total = 0;
   for (int l = 0; l < c->pol.n_layers; ++l) {
     if (layer >= 0 && l != layer) continue;
@@ -618,8 +639,8 @@ hwkv_status hwkv_allocated_ring_bytes(const hwkv_cache* c, int32_t layer, uint64
   uint64_t total = 0;
   for (int l = 0; l < c->pol.n_layers; ++l) {
     if (layer >= 0 && l != layer) continue;
-    for (int h = 0; h < H; ++h)
-      total += (uint64_t)c->lay.units[(size_t)l * H + h].cap * c->pol.head_dim * 4 *
+    for (int h = 0; h < H; ++h)  // rows held for the ring (codes and scales in 8 bits)
+      total += (uint64_t)c->lay.units[(size_t)l * H + h].stride * c->token_bytes() *
                (uint64_t)c->pol.batch;
   }
   *bytes = total;
@@ -653,13 +674,31 @@ hwkv_status hwkv_debug_copy_ring(const hwkv_cache* c, int32_t layer, int32_t b, 
       !v_host)
     return fail(HWKV_EINVAL, "bad ring coordinates or NULL buffer");
   const Unit& u = c->lay.units[(size_t)layer * c->pol.n_kv_heads + kv_head];
-  const size_t row = (size_t)c->pol.head_dim * 2;
-  const uint8_t* kb = c->arena + (size_t)(u.k_row0 + (int64_t)b * u.cap) * row;
-  const uint8_t* vb = c->arena + (size_t)(u.v_row0 + (int64_t)b * u.cap) * row;
+  const size_t row = (size_t)c->pol.head_dim * c->elem_bytes();
+  const uint8_t* kb = c->arena + (size_t)(u.k_row0 + (int64_t)b * u.stride) * row;
+  const uint8_t* vb = c->arena + (size_t)(u.v_row0 + (int64_t)b * u.stride) * row;
   cudaError_t e = cudaDeviceSynchronize();
   if (e == cudaSuccess) e = cudaMemcpy(k_host, kb, (size_t)u.cap * row, cudaMemcpyDeviceToHost);
   if (e == cudaSuccess) e = cudaMemcpy(v_host, vb, (size_t)u.cap * row, cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "ring copy: %s", cudaGetErrorString(e));
+  return ok();
+}
+
+hwkv_status hwkv_debug_copy_scales(const hwkv_cache* c, int32_t layer, int32_t b, int32_t kv_head,
+                                   float* k_scales, float* v_scales) {
+  hwkv_status st = check_layer(c, layer);
+  if (st != HWKV_OK) return st;
+  if (!c->fp8()) return fail(HWKV_EINVAL, "the cache is not in the 8-bit format");
+  if (b < 0 || b >= c->pol.batch || kv_head < 0 || kv_head >= c->pol.n_kv_heads || !k_scales ||
+      !v_scales)
+    return fail(HWKV_EINVAL, "bad ring coordinates or NULL buffer");
+  const Unit& u = c->lay.units[(size_t)layer * c->pol.n_kv_heads + kv_head];
+  const float* ks = c->scales() + u.k_row0 + (int64_t)b * u.stride;
+  const float* vs = c->scales() + u.v_row0 + (int64_t)b * u.stride;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpy(k_scales, ks, (size_t)u.cap * 4, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemcpy(v_scales, vs, (size_t)u.cap * 4, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "scale copy: %s", cudaGetErrorString(e));
   return ok();
 }
 
@@ -751,7 +790,7 @@ hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q,
   p.plan = reinterpret_cast<int64_t*>(scratch + o_bytes + ml_bytes);
   p.out = out;
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  e = launch_decode(p, c->kv_map, c->kv_map, d, grid, s);
+  e = launch_decode(p, c->kv_map, c->kv_map, d, grid, s, c->fp8());
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
   e = launch_decode_combine(p, d, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
