@@ -90,6 +90,31 @@ def lib():
             ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
             ctypes.c_void_p]
         L.oracle_ring_expected_fp8_gen.restype = ctypes.c_int
+        L.oracle_sink_visible.argtypes = [ctypes.c_int64] * 4
+        L.oracle_sink_visible.restype = ctypes.c_int
+        L.oracle_sink_positions.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                            ctypes.c_void_p]
+        L.oracle_sink_positions.restype = ctypes.c_int64
+        L.oracle_sink_attention_gen.argtypes = [
+            ctypes.POINTER(GenDesc), ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int64,
+            ctypes.c_int64, ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p]
+        L.oracle_sink_attention_gen.restype = ctypes.c_int
+        L.oracle_sink_attention_bf16.argtypes = [
+            ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p,
+            ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+            ctypes.c_int64, ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p]
+        L.oracle_sink_attention_bf16.restype = ctypes.c_int
+        L.oracle_sink_ring_positions.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                                 ctypes.c_void_p]
+        L.oracle_sink_ring_positions.restype = ctypes.c_int
+        L.oracle_sink_ring_expected_gen.argtypes = [
+            ctypes.POINTER(GenDesc), ctypes.c_uint32, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+            ctypes.c_void_p]
+        L.oracle_sink_ring_expected_gen.restype = ctypes.c_int
+        L.oracle_sink_retained_tokens.argtypes = [ctypes.c_int64] * 3
+        L.oracle_sink_retained_tokens.restype = ctypes.c_int64
         _lib = L
     return _lib
 
@@ -302,3 +327,66 @@ def ring_expected_fp8_gen(g, tensor, layer, b, kvh, d, t, cap):
                                           _p(codes), _p(scales)) != 0:
         raise ValueError("bad ring arguments")
     return codes, scales
+
+
+# ------------------------------------------------------- sink + recent window
+# The static sink--recent policy of the StreamingLLM control (App. baseline
+# controls): S sink tokens plus a W-token recent window.
+
+def sink_visible(k, p, W, S):
+    return bool(lib().oracle_sink_visible(k, p, W, S))
+
+
+def sink_positions(p, W, S):
+    """J of a query at p, increasing."""
+    n = int(lib().oracle_sink_positions(p, W, S, None))
+    out = np.zeros(max(n, 1), dtype=np.int64)
+    lib().oracle_sink_positions(p, W, S, _p(out))
+    return out[:n]
+
+
+def sink_attention_gen(g, layer, b, kvh, qheads, pos, d, W, S, gamma):
+    qh = np.ascontiguousarray(qheads, dtype=np.int32)
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    R = len(pos)
+    O = np.zeros((R, d))
+    sp = np.zeros(R)
+    rc = lib().oracle_sink_attention_gen(ctypes.byref(g), layer, b, kvh, _p(qh), _p(pos), R, d,
+                                         int(W), int(S), float(gamma), _p(O), _p(sp))
+    if rc != 0:
+        raise ValueError("oracle_sink_attention_gen failed (%d)" % rc)
+    return O, sp
+
+
+def sink_attention_bf16(Q, pos, Kp, Vp, W, S, gamma):
+    Q = np.ascontiguousarray(Q, dtype=np.uint16)
+    Kp = np.ascontiguousarray(Kp, dtype=np.uint16)
+    Vp = np.ascontiguousarray(Vp, dtype=np.uint16)
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    R, d = Q.shape
+    O = np.zeros((R, d))
+    sp = np.zeros(R)
+    rc = lib().oracle_sink_attention_bf16(_p(Q), d, _p(pos), R, _p(Kp), _p(Vp), d, Kp.shape[0], d,
+                                          int(W), int(S), float(gamma), _p(O), _p(sp))
+    if rc != 0:
+        raise ValueError("oracle_sink_attention_bf16 failed (%d)" % rc)
+    return O, sp
+
+
+def sink_ring_positions(t, W, S):
+    out = np.zeros(S + W, dtype=np.int64)
+    if lib().oracle_sink_ring_positions(t, W, S, _p(out)) != 0:
+        raise ValueError("bad ring arguments")
+    return out
+
+
+def sink_ring_expected_gen(g, tensor, layer, b, kvh, d, t, W, S):
+    out = np.zeros((S + W, d), dtype=np.uint16)
+    if lib().oracle_sink_ring_expected_gen(ctypes.byref(g), tensor, layer, b, kvh, d, t, W, S,
+                                           _p(out)) != 0:
+        raise ValueError("bad ring arguments")
+    return out
+
+
+def sink_retained_tokens(W, S, C):
+    return int(lib().oracle_sink_retained_tokens(W, S, C))

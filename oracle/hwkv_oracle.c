@@ -37,6 +37,14 @@
  *                       cache reads the dequantised rows (Sec. 3.1: when the format
  *                       changes execution, every compared output uses it).
  *
+ *   - sink + recent window (the static sink--recent policy of the StreamingLLM
+ *                       control the paper compares against, App. baseline controls:
+ *                       S sink tokens and a W-token recent window): a query at p
+ *                       reads J = {0..S-1} U [max(0, p-W+1), p], both limited to
+ *                       <= p; it retains min(S + W, C) tokens; held in a ring of
+ *                       S + W slots: positions < S in slots 0..S-1 for good, later
+ *                       ones in slot S + (p - S) mod W.
+ *
  * Windows are int64: 0 (HWKV_WINDOW_FULL) means full history; any W >= the
  * context is equivalent to full (Sec. 3.1). bf16 inputs are widened exactly to
  * double. Row loops may run under OpenMP; each row is computed independently.
@@ -253,6 +261,157 @@ int oracle_ring_expected_gen(const hwkv_gen_desc* g, uint32_t tensor, int32_t la
                                                    (uint32_t)kvh, (uint64_t)pos[j], (uint32_t)i, s);
   free(pos);
   return 0;
+}
+
+/* ------------------------------------------------------ sink + recent window */
+
+/* 1 if a query at position p reads key position k under window W (0 = full) with
+ * S sink tokens: k <= p and (k < S or k >= p - W + 1) */
+int oracle_sink_visible(int64_t k, int64_t p, int64_t W, int64_t S) {
+  if (k < 0 || k > p) return 0;
+  if (W == ORACLE_FULL) return 1;
+  return k < S || k >= p - W + 1;
+}
+
+/* the positions of J in increasing order: [0, min(S, p+1)) then [max(S, lo), p];
+ * returns their count (out may be NULL) */
+int64_t oracle_sink_positions(int64_t p, int64_t W, int64_t S, int64_t* out) {
+  if (p < 0) return 0;
+  const int64_t lo = oracle_window_lo(p, W);
+  const int64_t s_end = S < p + 1 ? S : p + 1;
+  int64_t n = 0;
+  for (int64_t k = 0; k < s_end; ++k) {
+    if (out) out[n] = k;
+    ++n;
+  }
+  for (int64_t k = (lo > s_end ? lo : s_end); k <= p; ++k) {
+    if (out) out[n] = k;
+    ++n;
+  }
+  return n;
+}
+
+/*
+ * Attention (Eq. conditional-attention-weight, Eq. conditional-attention) over J
+ * of the sink + recent policy, with q, K, V regenerated from the seeded generator:
+ * query rows (batch row b, query head qh[r], position pos[r]) reading KV head kvh.
+ */
+int oracle_sink_attention_gen(const hwkv_gen_desc* g, int32_t layer, int32_t b, int32_t kvh,
+                              const int32_t* qh, const int64_t* pos, int64_t R, int32_t d,
+                              int64_t W, int64_t S, double gamma, double* O, double* sum_pi) {
+  if (!g || R < 0 || d <= 0 || W < 0 || S < 0) return 1;
+  int bad = 0;
+  const float sk = hwkv_gen_head_scale(g, HWKV_GEN_K, (uint32_t)layer, (uint32_t)kvh);
+  const float sv = hwkv_gen_head_scale(g, HWKV_GEN_V, (uint32_t)layer, (uint32_t)kvh);
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t r = 0; r < R; ++r) {
+    const int64_t p = pos[r];
+    const int64_t n = oracle_sink_positions(p, W, S, NULL);
+    int64_t* J = (int64_t*)malloc(sizeof(int64_t) * (size_t)(n > 0 ? n : 1));
+    double* q = (double*)malloc(sizeof(double) * (size_t)d);
+    double* K = (double*)malloc(sizeof(double) * (size_t)(n * d + 1));
+    double* V = (double*)malloc(sizeof(double) * (size_t)(n * d + 1));
+    if (!J || !q || !K || !V || p < 0) {
+      bad = 1;
+    } else {
+      oracle_sink_positions(p, W, S, J);
+      const float sq = hwkv_gen_head_scale(g, HWKV_GEN_Q, (uint32_t)layer, (uint32_t)qh[r]);
+      for (int32_t i = 0; i < d; ++i)
+        q[i] = bf16_to_double(hwkv_gen_elem(g, HWKV_GEN_Q, (uint32_t)layer, (uint32_t)b,
+                                            (uint32_t)qh[r], (uint64_t)p, (uint32_t)i, sq));
+      for (int64_t j = 0; j < n; ++j)
+        for (int32_t i = 0; i < d; ++i) {
+          K[j * d + i] = bf16_to_double(hwkv_gen_elem(g, HWKV_GEN_K, (uint32_t)layer, (uint32_t)b,
+                                                      (uint32_t)kvh, (uint64_t)J[j], (uint32_t)i, sk));
+          V[j * d + i] = bf16_to_double(hwkv_gen_elem(g, HWKV_GEN_V, (uint32_t)layer, (uint32_t)b,
+                                                      (uint32_t)kvh, (uint64_t)J[j], (uint32_t)i, sv));
+        }
+      const double sp = oracle_attend(q, K, V, n, d, gamma, O + r * d, NULL);
+      if (sum_pi) sum_pi[r] = sp;
+    }
+    free(J);
+    free(q);
+    free(K);
+    free(V);
+  }
+  return bad ? 2 : 0;
+}
+
+/* The same over bf16 arrays indexed by absolute position (as
+ * oracle_window_attention_bf16). */
+int oracle_sink_attention_bf16(const uint16_t* Q, int64_t ldq, const int64_t* pos, int64_t R,
+                               const uint16_t* Kp, const uint16_t* Vp, int64_t ld, int64_t T,
+                               int64_t d, int64_t W, int64_t S, double gamma, double* O,
+                               double* sum_pi) {
+  if (R < 0 || d <= 0 || W < 0 || S < 0) return 1;
+  for (int64_t r = 0; r < R; ++r)
+    if (pos[r] < 0 || pos[r] >= T) return 1;
+  int bad = 0;
+  for (int64_t r = 0; r < R; ++r) {
+    const int64_t p = pos[r];
+    const int64_t n = oracle_sink_positions(p, W, S, NULL);
+    int64_t* J = (int64_t*)malloc(sizeof(int64_t) * (size_t)n);
+    double* q = (double*)malloc(sizeof(double) * (size_t)d);
+    double* K = (double*)malloc(sizeof(double) * (size_t)(n * d));
+    double* V = (double*)malloc(sizeof(double) * (size_t)(n * d));
+    if (!J || !q || !K || !V) {
+      bad = 1;
+    } else {
+      oracle_sink_positions(p, W, S, J);
+      for (int64_t i = 0; i < d; ++i) q[i] = bf16_to_double(Q[r * ldq + i]);
+      for (int64_t j = 0; j < n; ++j)
+        for (int64_t i = 0; i < d; ++i) {
+          K[j * d + i] = bf16_to_double(Kp[J[j] * ld + i]);
+          V[j * d + i] = bf16_to_double(Vp[J[j] * ld + i]);
+        }
+      const double sp = oracle_attend(q, K, V, n, d, gamma, O + r * d, NULL);
+      if (sum_pi) sum_pi[r] = sp;
+    }
+    free(J);
+    free(q);
+    free(K);
+    free(V);
+  }
+  return bad ? 2 : 0;
+}
+
+/*
+ * The ring of the sink + recent policy after positions 0..t-1 (cap = S + W
+ * slots, W > 0, S > 0): slot j < S holds position j once written; the window
+ * slots hold the latest W positions >= S, position p in slot S + (p - S) mod W.
+ * pos_of_slot[j] = the position held, or -1.
+ */
+int oracle_sink_ring_positions(int64_t t, int64_t W, int64_t S, int64_t* pos_of_slot) {
+  if (W <= 0 || S < 0 || t < 0) return 1;
+  for (int64_t j = 0; j < S + W; ++j) pos_of_slot[j] = -1;
+  for (int64_t p = 0; p < t && p < S; ++p) pos_of_slot[p] = p;
+  const int64_t first = t - W > S ? t - W : S;
+  for (int64_t p = first; p < t; ++p) pos_of_slot[S + (p - S) % W] = p;
+  return 0;
+}
+
+int oracle_sink_ring_expected_gen(const hwkv_gen_desc* g, uint32_t tensor, int32_t layer,
+                                  int32_t b, int32_t kvh, int32_t d, int64_t t, int64_t W,
+                                  int64_t S, uint16_t* ring) {
+  if (!g || W <= 0 || S < 0 || t < 0 || d <= 0) return 1;
+  const int64_t cap = S + W;
+  int64_t* pos = (int64_t*)malloc(sizeof(int64_t) * (size_t)cap);
+  if (!pos) return 2;
+  oracle_sink_ring_positions(t, W, S, pos);
+  const float s = hwkv_gen_head_scale(g, tensor, (uint32_t)layer, (uint32_t)kvh);
+  for (int64_t j = 0; j < cap; ++j)
+    for (int32_t i = 0; i < d; ++i)
+      ring[j * d + i] = pos[j] < 0 ? (uint16_t)0
+                                   : hwkv_gen_elem(g, tensor, (uint32_t)layer, (uint32_t)b,
+                                                   (uint32_t)kvh, (uint64_t)pos[j], (uint32_t)i, s);
+  free(pos);
+  return 0;
+}
+
+/* retained tokens of the sink + recent policy at context C: min(S + W, C); full: C */
+int64_t oracle_sink_retained_tokens(int64_t W, int64_t S, int64_t C) {
+  if (W == ORACLE_FULL) return C;
+  return S + W < C ? S + W : C;
 }
 
 /* ------------------------------------------------------- 8-bit KV format */
