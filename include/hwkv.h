@@ -79,6 +79,12 @@ typedef enum {
  *   windows[l * n_kv_heads + h] = W_{lh} in tokens (> 0), or HWKV_WINDOW_FULL.
  * A head with W >= max_ctx is stored as full. max_ctx bounds the tokens any
  * layer will ever hold (it is the ring capacity of full heads).
+ *   sinks: NULL, or sinks[l * n_kv_heads + h] = S >= 0 sink tokens kept beside a
+ *   finite window W (the static sink--recent policy of the paper's StreamingLLM
+ *   control): a query at position p then reads positions {0..S-1} and
+ *   [max(0, p-W+1), p] (both <= p), and the head retains min(S + W, t) tokens in
+ *   a ring of S + W slots (positions < S in slots 0..S-1 for good, later ones in
+ *   slot S + (p - S) mod W). Ignored for full heads; S + W >= max_ctx is full.
  * Supported: head_dim in {64, 128, 256}; n_q_heads / n_kv_heads <= 8;
  * batch <= 256; n_kv_heads <= 64; the policy is copied by hwkv_alloc.
  */
@@ -91,6 +97,7 @@ typedef struct {
   int32_t kv_format; /* HWKV_KV_BF16 or HWKV_KV_FP8_E4M3 */
   int64_t max_ctx;
   const int64_t* windows;
+  const int64_t* sinks; /* NULL: no sink tokens */
 } hwkv_policy;
 
 typedef struct hwkv_cache hwkv_cache; /* opaque; owned by the library */

@@ -35,17 +35,21 @@ class hwkv_policy(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
                 ("n_q_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("batch", ctypes.c_int32), ("kv_format", ctypes.c_int32),
-                ("max_ctx", ctypes.c_int64), ("windows", ctypes.POINTER(ctypes.c_int64))]
+                ("max_ctx", ctypes.c_int64), ("windows", ctypes.POINTER(ctypes.c_int64)),
+                ("sinks", ctypes.POINTER(ctypes.c_int64))]
 
 
 def make_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, max_ctx, windows,
-                kv_format=HWKV_KV_BF16):
+                kv_format=HWKV_KV_BF16, sinks=None):
     """hwkv_policy with its windows array ([n_layers * n_kv_heads] int64, 0 = full)
-    kept alive on the returned object."""
+    and optional sink counts (same shape) kept alive on the returned object."""
     w = np.ascontiguousarray(np.asarray(windows, dtype=np.int64).ravel())
+    sk = None if sinks is None else np.ascontiguousarray(np.asarray(sinks, dtype=np.int64).ravel())
     pol = hwkv_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, kv_format, max_ctx,
-                      w.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)))
+                      w.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+                      None if sk is None else sk.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)))
     pol._windows_keepalive = w
+    pol._sinks_keepalive = sk
     return pol
 
 

@@ -2,10 +2,10 @@
 // only its latest W states; App. "Runtime Realization": a head writes only its
 // own slice).
 //
-// Position p of KV head u goes to slot p mod cap_u; every row has its own
-// first position t0 (ragged rows). Of the n new tokens only the last
-// min(n, cap_u) are written: an earlier one would be overwritten in the same
-// call. Block 0 also stores the rows' new lengths in the device length array. One launch covers every KV head and batch row of a layer;
+// Position p of KV head u goes to slot p mod cap_u (with S sink slots: p < S
+// to slot p, later ones to slot S + (p - S) mod (cap_u - S)); every row has its
+// own first position t0 (ragged rows). A new token whose window slot a later
+// token of the same call takes is not written. Block 0 also stores the rows' new lengths in the device length array. One launch covers every KV head and batch row of a layer;
 // each thread moves one 16-byte vector, reads are coalesced over the input
 // [batch][n][heads][d] and writes over the ring rows.
 #include "hwkv_internal.cuh"
@@ -29,9 +29,10 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
     const int64_t i = r % p.n;
     const int b = (int)(r / p.n);
     const AppendUnit& u = p.u[h];
-    const int64_t keep = p.n < u.cap ? p.n : u.cap;
-    if (i < p.n - keep) continue;  // overwritten within this call
-    const int64_t slot = ((int64_t)p.t0[b] + i) % u.cap;
+    const int64_t pos = (int64_t)p.t0[b] + i;
+    // a window slot is overwritten within this call if position pos + (cap - sink) comes too
+    if (pos >= u.sink && pos < (int64_t)p.t0[b] + p.n - (u.cap - u.sink)) continue;
+    const int64_t slot = ring_slot(pos, u.cap, u.sink);
     const int64_t src = ((((int64_t)b * p.n + i) * p.n_units + h) * p.d) + vec * 8;
     const int64_t krow = u.k_row0 + (int64_t)(p.row0 + b) * u.stride + slot;
     const int64_t vrow = u.v_row0 + (int64_t)(p.row0 + b) * u.stride + slot;
@@ -63,9 +64,9 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
     const int64_t i = r % p.n;
     const int b = (int)(r / p.n);
     const AppendUnit& u = p.u[h];
-    const int64_t keep = p.n < u.cap ? p.n : u.cap;
-    if (i < p.n - keep) continue;  // overwritten within this call
-    const int64_t slot = ((int64_t)p.t0[b] + i) % u.cap;
+    const int64_t pos = (int64_t)p.t0[b] + i;
+    if (pos >= u.sink && pos < (int64_t)p.t0[b] + p.n - (u.cap - u.sink)) continue;
+    const int64_t slot = ring_slot(pos, u.cap, u.sink);
     const int64_t src = ((((int64_t)b * p.n + i) * p.n_units + h) * D) + lane * PER;
     const int64_t rows[2] = {u.k_row0 + (int64_t)(p.row0 + b) * u.stride + slot,
                              u.v_row0 + (int64_t)(p.row0 + b) * u.stride + slot};

@@ -245,7 +245,7 @@ struct TileWalker {
     ti.len = (int)len;
     ti.k_row = du.k_row0 + (int64_t)ti.b * du.stride + start;
     ti.v_row = du.v_row0 + (int64_t)ti.b * du.stride + start;
-    ti.s_new = (int64_t)len_b % du.cap;
+    ti.s_new = ring_slot(len_b, du.cap, du.sink);
     ti.single = start == 0 && len == n;
     ti.tile = 2 * (int)blockIdx.x + (first ? 0 : 1);
     rem -= len;

@@ -34,7 +34,13 @@ struct DecodeUnit {
   int64_t v_row0;   // same in the V region
   int64_t cap;      // ring capacity (slots)
   int64_t stride;   // rows between batch rows: batch row b starts at row0 + b * stride
+  int64_t sink;     // sink slots: positions < sink stay in slots 0..sink-1
 };
+
+// ring slot of position p: sinks first, then the window region of cap - sink slots
+__host__ __device__ __forceinline__ int64_t ring_slot(int64_t p, int64_t cap, int64_t sink) {
+  return p < sink ? p : sink + (p - sink) % (cap - sink);
+}
 
 // a tile of explicit key rows (SeqCalib replay): rows k_row.. / v_row.. of the trace
 // maps, queries of row q_row of q, KV head h
@@ -88,7 +94,7 @@ struct CalibCombineParams {
 
 // ------------------------------------------------------------------ append
 struct AppendUnit {
-  int64_t k_row0, v_row0, cap, stride;
+  int64_t k_row0, v_row0, cap, stride, sink;
 };
 
 struct AppendParams {
@@ -111,6 +117,7 @@ struct PrefillUnit {
   int64_t k_row0, v_row0, cap;
   int64_t window;  // 0 = full
   int64_t stride;  // rows between batch rows
+  int64_t sink;    // sink slots before the window region
 };
 
 struct PrefillParams {

@@ -68,62 +68,77 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
-// The key tiles one query block needs, in order: ring slot tiles whose newest
-// held position reaches the block's lowest visible key, then chunk tiles up to
-// the block's last row. Every role walks the same sequence.
+// The key tiles one query block needs, in order: the sink slots (all read by
+// every row), then tiles of the window region (slots S .. cap-1, positions >= S,
+// position p in slot S + (p - S) mod Wr) whose newest held position reaches the
+// block's lowest visible key, then chunk tiles up to the block's last row (from
+// the chunk's start while it still holds sink positions). A ring tile's j0 is its
+// first ring slot. Every role walks the same sequence. Without sinks (S = 0) the
+// window region is the whole ring.
 template <int BN>
 struct KeySeq {
-  int64_t t0, n, W, cap, n_hist, r0, lo_need, c_first, n_chunk_tiles, n_hist_tiles;
-  bool hist_needed;
-  int64_t hist_cur, chunk_cur;
+  int64_t t0, n, W, S, Wr, n_sink, tw, n_win, r0, lo_need, c_first, n_chunk_tiles;
+  int64_t n_sink_tiles, n_win_tiles;
+  bool win_needed;
+  int64_t sink_cur, win_cur, chunk_cur;
 
   __device__ void init(const PrefillUnit& u, int64_t t0_, int64_t n_, int64_t p0, int64_t p_last) {
     t0 = t0_;
     n = n_;
     W = u.window;
-    cap = u.cap;
-    n_hist = t0 < cap ? t0 : cap;
-    r0 = t0 % cap;
+    S = u.sink;
+    Wr = u.cap - S;
+    n_sink = t0 < S ? t0 : S;
+    tw = t0 > S ? t0 - S : 0;            // history tokens in the window region
+    n_win = tw < Wr ? tw : Wr;
+    r0 = tw % Wr;
     lo_need = W == 0 ? 0 : (p0 - W + 1 > 0 ? p0 - W + 1 : 0);
-    n_hist_tiles = (n_hist + BN - 1) / BN;
-    const int64_t c_lo = (t0 > lo_need ? t0 : lo_need) - t0;
+    n_sink_tiles = (n_sink + BN - 1) / BN;
+    n_win_tiles = (n_win + BN - 1) / BN;
+    // chunk keys below S are sinks, read by every row
+    const int64_t c_lo = t0 < S ? 0 : (t0 > lo_need ? t0 : lo_need) - t0;
     c_first = (c_lo / BN) * BN;
     const int64_t c_hi = p_last - t0;
     n_chunk_tiles = c_hi >= c_first ? (c_hi - c_first) / BN + 1 : 0;
-    hist_needed = n_hist > 0 && (W == 0 || p0 - W + 1 < t0);
-    hist_cur = next_hist(0);
+    win_needed = n_win > 0 && (W == 0 || p0 - W + 1 < t0);
+    sink_cur = 0;
+    win_cur = next_win(0);
     chunk_cur = 0;
   }
+  // position held by window-region slot j (0-based within the region)
   __device__ int64_t slot_pos(int64_t j) const {
-    if (t0 <= cap) return j;
-    return j < r0 ? t0 - r0 + j : t0 - r0 - cap + j;
+    if (tw <= Wr) return S + j;
+    return S + (j < r0 ? tw - r0 + j : tw - r0 - Wr + j);
   }
-  // smallest and largest position held in ring slots [j0, j1] (j1 < n_hist)
-  __device__ int64_t tile_min_pos(int64_t j0, int64_t j1) const {
-    if (t0 > cap && j0 < r0 && r0 <= j1) return slot_pos(r0);
-    return slot_pos(j0);
-  }
+  // largest position held in window-region slots [j0, j1] (j1 < n_win)
   __device__ int64_t tile_max_pos(int64_t j0, int64_t j1) const {
-    if (t0 > cap && j0 < r0 && r0 <= j1) return slot_pos(r0 - 1);
+    if (tw > Wr && j0 < r0 && r0 <= j1) return slot_pos(r0 - 1);
     return slot_pos(j1);
   }
-  __device__ bool ring_tile_needed(int64_t jt) const {
-    if (!hist_needed) return false;
+  __device__ bool win_tile_needed(int64_t jt) const {
+    if (!win_needed) return false;
     if (W == 0) return true;
     const int64_t j0 = jt * BN;
-    const int64_t j1 = (j0 + BN < n_hist ? j0 + BN : n_hist) - 1;
+    const int64_t j1 = (j0 + BN < n_win ? j0 + BN : n_win) - 1;
     return tile_max_pos(j0, j1) >= lo_need;
   }
-  __device__ int64_t next_hist(int64_t jt) const {
-    for (; jt < n_hist_tiles; ++jt)
-      if (ring_tile_needed(jt)) return jt;
+  __device__ int64_t next_win(int64_t jt) const {
+    for (; jt < n_win_tiles; ++jt)
+      if (win_tile_needed(jt)) return jt;
     return -1;
   }
+  // hist: 0 = chunk tile, 1 = window-region tile, 2 = sink tile
   __device__ bool next(int& hist, int64_t& j0) {
-    if (hist_cur >= 0) {
+    if (sink_cur < n_sink_tiles) {
+      hist = 2;
+      j0 = sink_cur * BN;
+      ++sink_cur;
+      return true;
+    }
+    if (win_cur >= 0) {
       hist = 1;
-      j0 = hist_cur * BN;
-      hist_cur = next_hist(hist_cur + 1);
+      j0 = S + win_cur * BN;
+      win_cur = next_win(win_cur + 1);
       return true;
     }
     if (chunk_cur < n_chunk_tiles) {
@@ -346,19 +361,27 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
       // columns e of this tile visible to row pr: [a0, b0) U [a1, b1)
       int a0 = 0, b0 = 0, a1 = 0, b1 = 0;
       if (row_ok) {
-        if (!hist) {  // chunk keys at positions t0 + j0 + e, held while j0 + e < n
+        if (hist == 0) {  // chunk keys at positions t0 + j0 + e, held while j0 + e < n
           const int64_t hi = min(pr - t0 - j0, p.n - 1 - j0);  // causal, held
           a0 = clampi(lo_r - t0 - j0);
           b0 = clampi(hi + 1);
-        } else if (t0 <= u.cap) {  // ring not yet wrapped: slot j holds position j
-          a0 = clampi(lo_r - j0);
-          b0 = clampi(seq.n_hist - j0);
-        } else {  // wrapped: slots < r0 hold the newest run, slots >= r0 the older one
-          const int64_t A = lo_r - t0 + seq.r0;  // first visible slot of the newest run
-          a0 = clampi(A - j0);
-          b0 = clampi(seq.r0 - j0);
-          a1 = clampi(A + u.cap - j0);
-          b1 = clampi(u.cap - j0);
+          b1 = clampi(min(seq.S - t0 - j0, hi + 1));  // chunk keys that are sinks
+        } else if (hist == 2) {  // sink slots: slot j holds position j, always visible
+          b0 = clampi(seq.n_sink - j0);
+        } else {
+          // window region, slots relative to its start: position S + v in slot
+          // S + (v mod Wr) for the region's v-th held token
+          const int64_t jw = j0 - seq.S, lo_v = lo_r - seq.S;
+          if (seq.tw <= seq.Wr) {  // not yet wrapped
+            a0 = clampi(lo_v - jw);
+            b0 = clampi(seq.n_win - jw);
+          } else {  // wrapped: slots < r0 hold the newest run, slots >= r0 the older one
+            const int64_t A = lo_v - seq.tw + seq.r0;  // first visible slot of the newest run
+            a0 = clampi(A - jw);
+            b0 = clampi(seq.r0 - jw);
+            a1 = clampi(A + seq.Wr - jw);
+            b1 = clampi(seq.Wr - jw);
+          }
         }
       }
       const bool full_vis = (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);

@@ -50,6 +50,7 @@ struct Unit {
   int64_t window;  // effective: 0 = full
   int64_t cap;
   int64_t stride;  // rows per batch row: cap, rounded up to 64 in the 8-bit format
+  int64_t sink;    // sink slots (sink + recent policy), 0 otherwise
   int64_t k_row0, v_row0;
 };
 
@@ -71,10 +72,14 @@ hwkv_status validate(const hwkv_policy* p) {
     return fail(HWKV_EINVAL, "n_q_heads (%d) must be a multiple of n_kv_heads (%d)",
                 p->n_q_heads, p->n_kv_heads);
   if (!p->windows) return fail(HWKV_EINVAL, "policy windows is NULL");
-  for (int64_t i = 0; i < (int64_t)p->n_layers * p->n_kv_heads; ++i)
+  for (int64_t i = 0; i < (int64_t)p->n_layers * p->n_kv_heads; ++i) {
     if (p->windows[i] < 0)
       return fail(HWKV_EINVAL, "window of (layer %lld, kv head %lld) is negative",
                   (long long)(i / p->n_kv_heads), (long long)(i % p->n_kv_heads));
+    if (p->sinks && p->sinks[i] < 0)
+      return fail(HWKV_EINVAL, "sink count of (layer %lld, kv head %lld) is negative",
+                  (long long)(i / p->n_kv_heads), (long long)(i % p->n_kv_heads));
+  }
   if (p->head_dim != 64 && p->head_dim != 128 && p->head_dim != 256)
     return fail(HWKV_EUNSUPPORTED, "head_dim %d not built (64, 128, 256)", p->head_dim);
   if (p->n_q_heads / p->n_kv_heads > kMaxGroup)
@@ -95,9 +100,12 @@ Layout make_layout(const hwkv_policy* p) {
   L.units.resize(nu);
   for (int i = 0; i < nu; ++i) {
     const int64_t W = p->windows[i];
+    const int64_t S = p->sinks ? p->sinks[i] : 0;
     Unit& u = L.units[i];
-    u.window = (W == HWKV_WINDOW_FULL || W >= p->max_ctx) ? 0 : W;  // w >= C is full (Sec. 3.1)
-    u.cap = u.window == 0 ? p->max_ctx : u.window;
+    // w >= C is full (Sec. 3.1); so is a sink + window that covers max_ctx
+    u.window = (W == HWKV_WINDOW_FULL || W >= p->max_ctx || S + W >= p->max_ctx) ? 0 : W;
+    u.sink = u.window == 0 ? 0 : S;
+    u.cap = u.window == 0 ? p->max_ctx : u.sink + u.window;
     // 8-bit rings start on 64-row boundaries: a stage's 64 scales are one aligned run
     u.stride = p->kv_format == HWKV_KV_FP8_E4M3 ? (u.cap + 63) / 64 * 64 : u.cap;
   }
@@ -150,7 +158,7 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 
 struct hwkv_cache {
   hwkv_policy pol;
-  std::vector<int64_t> windows;
+  std::vector<int64_t> windows, sinks;
   Layout lay;
   // tokens held per (layer, row), -1 = idle row: the host copy of the device
   // length array. A layer that has had a graph-mode step is advanced on the
@@ -230,6 +238,10 @@ hwkv_status hwkv_alloc(const hwkv_policy* policy, void* dev_arena, size_t arena_
   c->pol = *policy;
   c->windows.assign(policy->windows, policy->windows + (size_t)policy->n_layers * policy->n_kv_heads);
   c->pol.windows = c->windows.data();
+  if (policy->sinks) {
+    c->sinks.assign(policy->sinks, policy->sinks + (size_t)policy->n_layers * policy->n_kv_heads);
+    c->pol.sinks = c->sinks.data();
+  }
   c->lay = std::move(lay);
   c->t.assign((size_t)policy->n_layers * policy->batch, 0);
   c->dev_owned.assign(policy->n_layers, 0);
@@ -340,7 +352,7 @@ static AppendParams append_params(const hwkv_cache* c, int32_t layer, int32_t ro
   p.scales = c->scales();
   for (int h = 0; h < p.n_units; ++h) {
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
-    p.u[h] = AppendUnit{u.k_row0, u.v_row0, u.cap, u.stride};
+    p.u[h] = AppendUnit{u.k_row0, u.v_row0, u.cap, u.stride, u.sink};
   }
   return p;
 }
@@ -417,7 +429,7 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
   p.err = c->err();
   for (int h = 0; h < p.n_units; ++h) {
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
-    p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window, u.stride};
+    p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window, u.stride, u.sink};
   }
   // tensor maps of this call's q and chunk K/V: 3-D views {d, heads, batch * n}
   auto encode = get_encode();
@@ -509,7 +521,7 @@ static void ring_params(const hwkv_cache* c, int32_t layer, DecodeParams& p, int
   p.seg_cost = std::max(1, (int)((256 << 10) / c->token_bytes() / kStageTokens));
   for (int h = 0; h < p.n_units; ++h) {
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
-    p.u[h] = DecodeUnit{u.k_row0, u.v_row0, u.cap, u.stride};
+    p.u[h] = DecodeUnit{u.k_row0, u.v_row0, u.cap, u.stride, u.sink};
   }
 }
 
