@@ -278,17 +278,16 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 }
 
 // FP8: K/V stages hold E4M3 codes (one byte per channel, 128 channels per
-// 128-byte slab) and each stage's 64 K and 64 V row scales arrive beside it; every
-// consumer warp dequantises its 16 V rows into a private f16 scratch.
+// 128-byte slab) and each stage's 64 K and 64 V row scales arrive beside it.
 template <int D, bool FP8>
 struct DecodeCfg {
   static constexpr int kChanPerSlab = FP8 ? 128 : 64;
   static constexpr int kSlabs = D / kChanPerSlab;
   static constexpr int kTileBytes = kSlabs * kSlabBytes;  // 64 tokens of K (or V)
   static constexpr int kStageBytes = 2 * kTileBytes;
-  static constexpr int kStages = FP8 ? (D == 256 ? 4 : 8) : (D == 256 ? 3 : (D == 128 ? 6 : 8));
+  static constexpr int kStages = FP8 ? (D == 256 ? 5 : 10) : (D == 256 ? 3 : (D == 128 ? 6 : 8));
   static constexpr int kScaleBytes = FP8 ? kStages * 2 * kStageTokens * 4 : 0;
-  static constexpr int kScratchBytes = FP8 ? kDecodeWarps * 16 * D * 2 : 0;  // f16 V rows
+  static constexpr int kScratchBytes = 0;
   static constexpr int kRedLd = D + 4;  // padded row of the cross-warp merge area (floats)
   static constexpr int kRedBytes = kDecodeWarps * kMaxGroup * kRedLd * 4;
   static constexpr int kMlBytes = kDecodeWarps * kMaxGroup * 8;
@@ -306,9 +305,8 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
   constexpr int STAGES = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* scratch = smem + STAGES * C::kStageBytes;               // FP8: [warp][16 rows] f16
-  float* stage_scales = reinterpret_cast<float*>(scratch + C::kScratchBytes);  // [stage][K|V][64]
-  uint8_t* tail = scratch + C::kScratchBytes + C::kScaleBytes;
+  float* stage_scales = reinterpret_cast<float*>(smem + STAGES * C::kStageBytes);  // FP8: [stage][K|V][64]
+  uint8_t* tail = smem + STAGES * C::kStageBytes + C::kScaleBytes;
   float* red_o = reinterpret_cast<float*>(tail);
   float2* red_ml = reinterpret_cast<float2*>(tail + C::kRedBytes);
   uint64_t* full = reinterpret_cast<uint64_t*>(tail + C::kRedBytes + C::kMlBytes);
@@ -570,35 +568,6 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
         s1 *= ksA;
         s2 *= ksB;
         s3 *= ksB;
-        // dequantise this warp's 16 V rows into its f16 scratch (same swizzled layout
-        // as a bf16 V tile), then the stage can be refilled
-        const int rr = lane >> 1, hf = lane & 1;
-        const uint32_t sw = smem_u32(scratch) + w * (16 * D * 2);
-        constexpr int CH = D / 32;  // 16-byte E4M3 chunks per lane
-#pragma unroll
-        for (int j = 0; j < CH; ++j) {
-          const int g = hf * CH + j;  // channels 16g .. 16g + 15
-          uint32_t x0, x1, x2, x3;
-          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                       : "=r"(x0), "=r"(x1), "=r"(x2), "=r"(x3)
-                       : "r"(vbase + (g >> 3) * kSlabBytes + swz128(w * 16 + rr, g & 7))
-                       : "memory");
-          uint32_t f[8];
-          e4m3x4_to_f16x2(x0, f[0], f[1]);
-          e4m3x4_to_f16x2(x1, f[2], f[3]);
-          e4m3x4_to_f16x2(x2, f[4], f[5]);
-          e4m3x4_to_f16x2(x3, f[6], f[7]);
-          const uint32_t d0 = sw + (g >> 2) * (16 * 128) + swz128(rr, (g & 3) * 2);
-          const uint32_t d1 = sw + (g >> 2) * (16 * 128) + swz128(rr, (g & 3) * 2 + 1);
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(d0), "r"(f[0]), "r"(f[1]),
-                       "r"(f[2]), "r"(f[3])
-                       : "memory");
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(d1), "r"(f[4]), "r"(f[5]),
-                       "r"(f[6]), "r"(f[7])
-                       : "memory");
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[s]);
       }
       const int tok = st * kStageTokens + w * 16 + (lane >> 2);
       if (tok >= ti.len) s0 = s1 = -INFINITY;
@@ -646,19 +615,27 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
             mma_bf16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
           }
         } else {
-          const int rl = (lane & 7) + (mi >> 1) * 8;
-          const uint32_t sw = smem_u32(scratch) + w * (16 * D * 2);
+          // V^T fragments straight from the E4M3 stage: the transposing x4 load of
+          // byte pairs gives each lane tokens (2q, 2q+1) x channels (2g, 2g+1) of 16
+          // tokens x 32 channels; a byte permute splits them into the even- and
+          // odd-channel token pairs, which feed two f16 mmas (o[2kk]: channels
+          // 32kk + 2g (+16), o[2kk + 1]: the odd ones)
+          const int tr = w * 16 + (mi >> 1) * 8 + (lane & 7);
 #pragma unroll
-          for (int mt = 0; mt < D / 16; ++mt) {
-            uint32_t a0, a1, a2, a3;
-            ldsm_x4_t(sw + (mt >> 2) * (16 * 128) + swz128(rl, (mt & 3) * 2 + csel), a0, a1, a2,
-                      a3);
-            mma_f16_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+          for (int kk = 0; kk < D / 32; ++kk) {
+            const int ch = kk * 32 + (mi & 1) * 16;
+            uint32_t r[4], lo[4], hi[4];
+            ldsm_x4_t(vbase + (ch >> 7) * kSlabBytes + swz128(tr, (ch & 127) >> 4), r[0], r[1],
+                      r[2], r[3]);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) e4m3x4_to_f16x2(__byte_perm(r[j], 0, 0x3120), lo[j], hi[j]);
+            mma_f16_16816(o[2 * kk], lo[0], lo[1], lo[2], lo[3], pb0, pb1);
+            mma_f16_16816(o[2 * kk + 1], hi[0], hi[1], hi[2], hi[3], pb0, pb1);
           }
         }
       }
       __syncwarp();
-      if (!FP8 && lane == 0) mbar_arrive(&empty[s]);
+      if (lane == 0) mbar_arrive(&empty[s]);
     }
 
     // ---- merge the four warps' partials of this tile in shared memory
@@ -672,11 +649,14 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
       float* ro = red_o + (size_t)w * kMaxGroup * C::kRedLd;
 #pragma unroll
       for (int mt = 0; mt < D / 16; ++mt) {
-        const int dim = mt * 16 + (lane >> 2);
+        // bf16: o[mt] rows are channels 16 mt + g and + 8; FP8: 32 (mt / 2) + 2g + (mt & 1)
+        // and + 16 (the channel order of the V^T fragments)
+        const int dim = FP8 ? (mt >> 1) * 32 + 2 * (lane >> 2) + (mt & 1) : mt * 16 + (lane >> 2);
+        const int dim2 = dim + (FP8 ? 16 : 8);
         ro[qk * C::kRedLd + dim] = o[mt][0];
         ro[(qk + 1) * C::kRedLd + dim] = o[mt][1];
-        ro[qk * C::kRedLd + dim + 8] = o[mt][2];
-        ro[(qk + 1) * C::kRedLd + dim + 8] = o[mt][3];
+        ro[qk * C::kRedLd + dim2] = o[mt][2];
+        ro[(qk + 1) * C::kRedLd + dim2] = o[mt][3];
       }
       if (lane < 4) {
         red_ml[w * kMaxGroup + qk] = make_float2(mA, lA);
