@@ -51,7 +51,8 @@ typedef enum {
   HWKV_ECAPACITY = 3,    /* append would exceed max_ctx on a full-history head */
   HWKV_ECUDA = 4,        /* a CUDA runtime call or launch failed */
   HWKV_EKERNEL = 5,      /* a kernel reported an internal error (see hwkv_sync_check) */
-  HWKV_EUNSUPPORTED = 6  /* valid request outside the built kernel set (e.g. head_dim) */
+  HWKV_EUNSUPPORTED = 6, /* valid request outside the built kernel set (e.g. head_dim) */
+  HWKV_ETRACE = 7        /* hwkv_calib_trace_check: the trace does not match its replay */
 } hwkv_status;
 
 /* windows[] entry meaning "full history" (Sec. 3.1: a_{lh} = full) */
@@ -318,6 +319,24 @@ HWKV_API hwkv_status hwkv_calib_scores(const hwkv_calib_desc* desc, const void* 
                                        const void* v, float scale, void* workspace,
                                        size_t ws_bytes, double* scores, float* cos_out,
                                        void* cuda_stream);
+
+/*
+ * Trace-compatibility check of SeqCalib (App. "Experimental Protocol" and
+ * App. "Runtime Realization": before accepting a layer's trace the calibrator
+ * replays the full-window attention for the sampled positions and aborts the run
+ * when it does not reproduce the traced output; the paper aborts below cosine
+ * 0.99). Same replay as hwkv_calib_scores; traced: device fp32
+ * [N][P][n_q_heads][head_dim], the traced full-history outputs at the sampled
+ * positions. *min_cos receives the smallest cos_eval(replayed full, traced)
+ * (App. A.2, Eq. stabilized-cosine); trace_cos_out (host [N][P][n_q_heads] or
+ * NULL) all of them. Returns HWKV_ETRACE (naming the worst row) when
+ * *min_cos < threshold. Synchronizes `cuda_stream`.
+ */
+HWKV_API hwkv_status hwkv_calib_trace_check(const hwkv_calib_desc* desc, const void* q,
+                                            const void* k, const void* v, float scale,
+                                            const float* traced, double threshold,
+                                            void* workspace, size_t ws_bytes, double* min_cos,
+                                            float* trace_cos_out, void* cuda_stream);
 
 /*
  * Threshold selection (Sec. 3.2, Eq. threshold-selection) for each of n_heads

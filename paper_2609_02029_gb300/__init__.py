@@ -18,11 +18,11 @@ LIB_PATH = os.path.join(_HERE, "libhwkv.so")
 HEADER = os.path.join(os.path.dirname(_HERE), "include", "hwkv.h")
 
 HWKV_OK, HWKV_EINVAL, HWKV_ENOMEM, HWKV_ECAPACITY = 0, 1, 2, 3
-HWKV_ECUDA, HWKV_EKERNEL, HWKV_EUNSUPPORTED = 4, 5, 6
+HWKV_ECUDA, HWKV_EKERNEL, HWKV_EUNSUPPORTED, HWKV_ETRACE = 4, 5, 6, 7
 HWKV_WINDOW_FULL = 0
 HWKV_KV_BF16, HWKV_KV_FP8_E4M3 = 0, 1
 STATUS_NAMES = {0: "HWKV_OK", 1: "HWKV_EINVAL", 2: "HWKV_ENOMEM", 3: "HWKV_ECAPACITY",
-                4: "HWKV_ECUDA", 5: "HWKV_EKERNEL", 6: "HWKV_EUNSUPPORTED"}
+                4: "HWKV_ECUDA", 5: "HWKV_EKERNEL", 6: "HWKV_EUNSUPPORTED", 7: "HWKV_ETRACE"}
 
 
 class HwkvError(RuntimeError):
@@ -113,6 +113,9 @@ def lib():
             "hwkv_calib_scores": [ctypes.POINTER(hwkv_calib_desc), _vp, _vp, _vp, ctypes.c_float,
                                   _vp, ctypes.c_size_t, _vp, _vp, _vp],
             "hwkv_calib_select": [_vp, _i32, _vp, _i32, _i64, ctypes.c_double, _vp],
+            "hwkv_calib_trace_check": [ctypes.POINTER(hwkv_calib_desc), _vp, _vp, _vp,
+                                       ctypes.c_float, _vp, ctypes.c_double, _vp, ctypes.c_size_t,
+                                       ctypes.POINTER(ctypes.c_double), _vp, _vp],
             "hwkv_budget_select": [_vp, _vp, _i32, ctypes.c_double, ctypes.POINTER(_i32)],
             "hwkv_policy_save": [ctypes.c_char_p, ctypes.c_char_p, ctypes.c_uint64, _i32, _i32, _vp],
             "hwkv_policy_load": [ctypes.c_char_p, ctypes.c_char_p, ctypes.c_size_t,
@@ -302,6 +305,18 @@ def hwkv_calib_scores(desc, q, k, v, scale, workspace, ws_bytes, stream=None, wi
                                    cos.ctypes.data_as(_vp) if cos is not None else None,
                                    _stream(stream)))
     return scores, cos
+
+
+def hwkv_calib_trace_check(desc, q, k, v, scale, traced, workspace, ws_bytes, threshold=0.99,
+                           stream=None):
+    """(min cosine, per-row cosines [N, P, n_q_heads]) of the replayed full-window
+    outputs against the traced ones; raises HwkvError(HWKV_ETRACE) below threshold."""
+    m = ctypes.c_double(0.0)
+    per = np.zeros((desc.n_seq, desc.n_pos, desc.n_q_heads), dtype=np.float32)
+    _check(lib().hwkv_calib_trace_check(ctypes.byref(desc), _ptr(q), _ptr(k), _ptr(v), scale,
+                                        _ptr(traced), threshold, _ptr(workspace), ws_bytes,
+                                        ctypes.byref(m), per.ctypes.data_as(_vp), _stream(stream)))
+    return m.value, per
 
 
 def hwkv_calib_select(scores, windows, C, tau):

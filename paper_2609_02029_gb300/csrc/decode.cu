@@ -854,7 +854,9 @@ cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& kmap, const 
 // merges the band partials of query head g in band order; after band k (< K)
 // the running output is o^(W_k), after the last band it is o^(full). Each
 // candidate is scored against full with the stabilized cosine (eps = 1e-12:
-// a vector of norm <= eps counts as zero; both zero -> 1, one zero -> 0).
+// a vector of norm <= eps counts as zero; both zero -> 1, one zero -> 0); with
+// a traced output given, o^(full) is scored against it the same way (the
+// calibrator's trace-compatibility check, App. "Experimental Protocol").
 constexpr int kCalibMaxWindows = 8;
 
 template <int D>
@@ -940,6 +942,25 @@ __global__ void __launch_bounds__(kMaxGroup * 32) calib_combine_kernel(const Cal
     const bool zu = nu <= 1e-12f, zf = nf <= 1e-12f;
     const float cv = (zu && zf) ? 1.f : ((zu || zf) ? 0.f : uv / (nu * nf));
     if (lane == 0) p.cos[((int64_t)u * p.group + g) * K + k] = cv;
+  }
+  if (p.traced != nullptr) {
+    // trace check: the replayed full-window output against the traced one
+    const float* tr = p.traced + ((int64_t)u * p.group + g) * D + lane * PER;
+    float tt = 0.f, ft = 0.f;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) {
+      tt += tr[e] * tr[e];
+      ft += tr[e] * full[e];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      tt += __shfl_xor_sync(0xffffffffu, tt, off);
+      ft += __shfl_xor_sync(0xffffffffu, ft, off);
+    }
+    const float nt = sqrtf(tt);
+    const bool zt = nt <= 1e-12f, zf = nf <= 1e-12f;
+    const float cv = (zt && zf) ? 1.f : ((zt || zf) ? 0.f : ft / (nt * nf));
+    if (lane == 0) p.trace_cos[(int64_t)u * p.group + g] = cv;
   }
 }
 

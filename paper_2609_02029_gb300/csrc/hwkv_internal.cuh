@@ -90,6 +90,8 @@ struct CalibCombineParams {
   const float* part_o;        // [tiles][kMaxGroup][D]
   const float2* part_ml;      // [tiles][kMaxGroup]
   float* cos;                 // [n_units][G][K]
+  const float* traced;        // NULL, or [n_units][G][D]: traced full-history outputs
+  float* trace_cos;           // with traced: [n_units][G] cos_eval(replayed full, traced)
 };
 
 // ------------------------------------------------------------------ append

@@ -839,7 +839,8 @@ struct CalibPlan {
   std::vector<CalibTile> tiles;
   std::vector<int32_t> band_begin;  // [units][K + 2]
   int64_t units = 0;
-  size_t off_tiles = 0, off_bands = 0, off_o = 0, off_ml = 0, off_cos = 0, off_err = 0, total = 0;
+  size_t off_tiles = 0, off_bands = 0, off_o = 0, off_ml = 0, off_cos = 0, off_tcos = 0;
+  size_t off_err = 0, total = 0;
 };
 
 // Nested-suffix bands of position t for increasing windows W[0..K-1]: band 0 =
@@ -881,7 +882,8 @@ static CalibPlan calib_plan(const hwkv_calib_desc* d) {
   P.off_o = align_up(P.off_bands + P.band_begin.size() * 4, kAlign);
   P.off_ml = align_up(P.off_o + nt * kMaxGroup * d->head_dim * 4, kAlign);
   P.off_cos = align_up(P.off_ml + nt * kMaxGroup * 8, kAlign);
-  P.off_err = align_up(P.off_cos + (size_t)P.units * G * K * 4, kAlign);
+  P.off_tcos = align_up(P.off_cos + (size_t)P.units * G * K * 4, kAlign);
+  P.off_err = align_up(P.off_tcos + (size_t)P.units * G * 4, kAlign);
   P.total = align_up(P.off_err + 64, kAlign);
   return P;
 }
@@ -894,12 +896,15 @@ hwkv_status hwkv_calib_workspace_bytes(const hwkv_calib_desc* d, size_t* bytes) 
   return ok();
 }
 
-hwkv_status hwkv_calib_scores(const hwkv_calib_desc* d, const void* q, const void* k,
-                              const void* v, float scale, void* workspace, size_t ws_bytes,
-                              double* scores, float* cos_out, void* cuda_stream) {
+// The replay shared by hwkv_calib_scores and hwkv_calib_trace_check: fills cosv
+// [units][G][K] and, with traced, tcos [units][G]; synchronizes the stream.
+static hwkv_status calib_run(const hwkv_calib_desc* d, const void* q, const void* k,
+                             const void* v, float scale, void* workspace, size_t ws_bytes,
+                             const float* traced, std::vector<float>& cosv,
+                             std::vector<float>& tcos, void* cuda_stream) {
   hwkv_status st = calib_validate(d);
   if (st != HWKV_OK) return st;
-  if (!q || !k || !v || !workspace || !scores) return fail(HWKV_EINVAL, "NULL argument");
+  if (!q || !k || !v || !workspace) return fail(HWKV_EINVAL, "NULL argument");
   if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
   const CalibPlan P = calib_plan(d);
   if (ws_bytes < P.total) return fail(HWKV_ENOMEM, "workspace %zu < required %zu", ws_bytes, P.total);
@@ -958,15 +963,31 @@ hwkv_status hwkv_calib_scores(const hwkv_calib_desc* d, const void* q, const voi
   cp.part_o = p.part_o;
   cp.part_ml = p.part_ml;
   cp.cos = reinterpret_cast<float*>(ws + P.off_cos);
+  cp.traced = traced;
+  cp.trace_cos = reinterpret_cast<float*>(ws + P.off_tcos);
   e = launch_calib_combine(cp, D, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "calib combine launch: %s", cudaGetErrorString(e));
-  std::vector<float> cosv((size_t)P.units * G * K);
+  cosv.assign((size_t)P.units * G * K, 0.f);
+  tcos.assign(traced ? (size_t)P.units * G : 0, 0.f);
   int err_word = 0;
   e = cudaMemcpyAsync(cosv.data(), cp.cos, cosv.size() * 4, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess && traced)
+    e = cudaMemcpyAsync(tcos.data(), cp.trace_cos, tcos.size() * 4, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(&err_word, p.err, sizeof(int), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "calib readback: %s", cudaGetErrorString(e));
   if (err_word != 0) return fail(HWKV_EKERNEL, "calib kernel error word 0x%x", err_word);
+  return HWKV_OK;
+}
+
+hwkv_status hwkv_calib_scores(const hwkv_calib_desc* d, const void* q, const void* k,
+                              const void* v, float scale, void* workspace, size_t ws_bytes,
+                              double* scores, float* cos_out, void* cuda_stream) {
+  if (!scores) return fail(HWKV_EINVAL, "scores is NULL");
+  std::vector<float> cosv, tcos;
+  hwkv_status st = calib_run(d, q, k, v, scale, workspace, ws_bytes, nullptr, cosv, tcos, cuda_stream);
+  if (st != HWKV_OK) return st;
+  const int H = d->n_kv_heads, G = d->n_q_heads / d->n_kv_heads, K = d->n_windows;
   // Eq. conditional-similarity: mean over (sequence, position, query head), fixed order
   const double inv = 1.0 / ((double)d->n_seq * d->n_pos * G);
   for (int h = 0; h < H; ++h)
@@ -982,6 +1003,34 @@ hwkv_status hwkv_calib_scores(const hwkv_calib_desc* d, const void* q, const voi
         for (int g = 0; g < G; ++g)
           for (int kk = 0; kk < K; ++kk)
             cos_out[((np * d->n_q_heads) + h * G + g) * K + kk] = cosv[((np * H + h) * G + g) * K + kk];
+  return ok();
+}
+
+hwkv_status hwkv_calib_trace_check(const hwkv_calib_desc* d, const void* q, const void* k,
+                                   const void* v, float scale, const float* traced,
+                                   double threshold, void* workspace, size_t ws_bytes,
+                                   double* min_cos, float* trace_cos_out, void* cuda_stream) {
+  if (!traced || !min_cos) return fail(HWKV_EINVAL, "traced/min_cos is NULL");
+  std::vector<float> cosv, tcos;
+  hwkv_status st = calib_run(d, q, k, v, scale, workspace, ws_bytes, traced, cosv, tcos, cuda_stream);
+  if (st != HWKV_OK) return st;
+  double m = 1.0;
+  int64_t worst = 0;
+  for (size_t i = 0; i < tcos.size(); ++i)
+    if ((double)tcos[i] < m) {
+      m = tcos[i];
+      worst = (int64_t)i;
+    }
+  *min_cos = m;
+  if (trace_cos_out) std::copy(tcos.begin(), tcos.end(), trace_cos_out);  // [N][P][n_q_heads]
+  if (m < threshold) {
+    const int64_t Hq = d->n_q_heads;
+    return fail(HWKV_ETRACE,
+                "trace check failed: replayed full-window output of (sequence %lld, position "
+                "index %lld, query head %lld) has cosine %.6f < %.3f against the trace",
+                (long long)(worst / Hq / d->n_pos), (long long)(worst / Hq % d->n_pos),
+                (long long)(worst % Hq), m, threshold);
+  }
   return ok();
 }
 

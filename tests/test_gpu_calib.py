@@ -78,3 +78,37 @@ def test_calib_scores_match_oracle(N, P, T, Hkv, Hq, d, windows):
         got = hwkv.hwkv_calib_select(scores, windows, T, tau)
         want = [oracle.select_window(want_scores[h], windows, T, tau) for h in range(Hkv)]
         assert list(got) == want
+
+
+def test_trace_check_accepts_matching_trace_and_rejects_wrong_mapping():
+    # the traced full-history outputs (here: the oracle's full-window attention) must be
+    # reproduced by the replay; a trace whose query heads read the wrong KV head (a GQA
+    # mapping mismatch) must fail the 0.99 check (App. "Experimental Protocol")
+    import torch
+    N, P, T, Hkv, Hq, d = 2, 4, 1500, 2, 8, 128
+    g = hwkv_gen.desc(23, per_head_scale=True)
+    pos = np.sort(np.random.default_rng(3).integers(T // 2, T, size=(N, P)), axis=1)
+    Qd, Kh, Vh, Q, Khost, Vhost = _trace(g, N, T, Hkv, Hq, d, pos)
+    G = Hq // Hkv
+    scale = 1.0 / np.sqrt(d)
+
+    def traced_outputs(kv_of_q):
+        out = np.zeros((N, P, Hq, d), dtype=np.float32)
+        for n in range(N):
+            for qh in range(Hq):
+                h = kv_of_q(qh)
+                O, _ = oracle.window_attention_bf16(Q[n, :, qh], pos[n], Khost[n, :, h],
+                                                    Vhost[n, :, h], 0, scale)
+                out[n, :, qh] = O
+        return torch.from_numpy(out).cuda()
+
+    desc = hwkv.make_calib_desc(N, P, Hkv, Hq, d, T, [64, 512], pos)
+    nbytes = hwkv.hwkv_calib_workspace_bytes(desc)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    m, per = hwkv.hwkv_calib_trace_check(desc, Qd, Kh, Vh, scale, traced_outputs(lambda q: q // G),
+                                         ws, nbytes)
+    assert m > 0.999 and per.min() == np.float32(m)
+    with pytest.raises(hwkv.HwkvError) as e:
+        hwkv.hwkv_calib_trace_check(desc, Qd, Kh, Vh, scale,
+                                    traced_outputs(lambda q: (q // G + 1) % Hkv), ws, nbytes)
+    assert e.value.status == hwkv.HWKV_ETRACE
