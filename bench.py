@@ -38,7 +38,7 @@ L2_BYTES = 129 * 1024 * 1024
 # capture (--set full) of the 1-layer, batch-2 case of layers16_112k;
 # traffic is reads of every resident K/V row plus tile partials, so it scales with the
 # algorithmic bytes of a launch. Set to None whenever that kernel changes.
-DECODE_TRAFFIC_PER_BYTE = (244.297472e6 + 4.015104e6) / 244066304.0
+DECODE_TRAFFIC_PER_BYTE = (244.301312e6 + 3.917312e6) / 244066304.0
 
 
 def peaks():

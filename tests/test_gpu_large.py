@@ -1,10 +1,11 @@
 """Full-size parity for the two large workloads, in the launch configuration
-bench.py times: the 112K-context, 16-layer, batch-16 decode (39 GB of rings)
-and the 161K-context budget sweep (25/50/75/100% of all-full residency, up to
-43 GB). The whole prompt is appended through the C ABI; decode steps run over
-every layer. Seeded samples of (layer, batch row, KV head) units are checked
-against the oracle at the first and last step, sampled rings bit-exactly, and
-residency exactly at every step."""
+bench.py times (hwkv_decode_step: the new token's append fused into the decode
+launch, work planned on the GPU): the 112K-context, 16-layer, batch-16 decode
+(39 GB of rings) and the 161K-context budget sweep (25/50/75/100% of all-full
+residency, up to 43 GB). The whole prompt is appended through the C ABI; decode
+steps run over every layer. Seeded samples of (layer, batch row, KV head) units
+are checked against the oracle at the first and last step, sampled rings
+bit-exactly, and residency exactly at every step."""
 import numpy as np
 import pytest
 
@@ -35,7 +36,7 @@ def _run_decode_workload(wl, steps, n_units, seed):
         torch.cuda.synchronize()
         units = _units(wl, rng, n_units)
         for step in range(steps):
-            outs = [r.decode_step(layer) for layer in range(wl.n_layers)]
+            outs = [r.decode_step_fused(layer) for layer in range(wl.n_layers)]
             t = wl.prompt + step + 1
             assert hwkv.hwkv_residency_bytes(r.cache) == oracle.nominal_storage(
                 wl.windows, t, wl.head_dim, wl.head_dim, 2, 2, wl.batch)
@@ -52,7 +53,7 @@ def _run_decode_workload(wl, steps, n_units, seed):
 
 
 def test_layers16_112k_decode():
-    _run_decode_workload(workloads.make("layers16_112k"), steps=3, n_units=14, seed=3)
+    _run_decode_workload(workloads.make("layers16_112k"), steps=3, n_units=24, seed=3)
 
 
 @pytest.mark.parametrize("budget", [0.25, 0.5, 0.75, 1.0])
