@@ -181,12 +181,18 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
+  // K and V tiles live in separate buffers, released separately: a K buffer as soon
+  // as its QK^T is done, a V buffer when its PV is done, so the next K tiles load
+  // while this tile's softmax and PV run
   uint8_t* sQ = smem;
-  uint8_t* sStage = smem + C::kQBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + STAGES * C::kStageBytes);
-  uint64_t* kv_full = bars;              // [STAGES] TMA landed
-  uint64_t* kv_empty = bars + STAGES;    // [STAGES] PV of that tile done
-  uint64_t* s_full = bars + 2 * STAGES;  // [2] S tile computed
+  uint8_t* sK = smem + C::kQBytes;                      // [STAGES] K tiles
+  uint8_t* sV = sK + STAGES * C::kTileBytes;            // [STAGES] V tiles
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sK + STAGES * C::kStageBytes);
+  uint64_t* k_full = bars;                // [STAGES] K tile landed
+  uint64_t* k_empty = bars + STAGES;      // [STAGES] QK^T of that tile done
+  uint64_t* v_full = bars + 2 * STAGES;   // [STAGES] V tile landed
+  uint64_t* v_empty = bars + 3 * STAGES;  // [STAGES] PV of that tile done
+  uint64_t* s_full = bars + 4 * STAGES;   // [2] S tile computed
   uint64_t* s_free = s_full + 2;         // [2] S tile read by the softmax warps
   uint64_t* p_full = s_free + 2;         // P of the current tile written (and O rescaled)
   uint64_t* pv_done = p_full + 1;        // PV mma of the previous tile done
@@ -211,8 +217,10 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
@@ -252,39 +260,46 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
         tma_load_3d(sQ + sl * C::kQSlab, &q_map, sl * 64, h * G, qrow, q_full);
       const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;
       const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.stride;
-      uint32_t it = 0;
-      int hist;
-      int64_t j0;
-      while (seq.next(hist, j0)) {
+      // two walks of the same key sequence: K tiles run one tile ahead of V tiles
+      KeySeq<BN> seq_v = seq;
+      uint32_t it_k = 0, it_v = 0;
+      auto issue = [&](KeySeq<BN>& sq, uint32_t& it, uint64_t* full, uint64_t* empty,
+                       uint8_t* buf, int64_t row0, const CUtensorMap* cmap) -> bool {
+        int hist;
+        int64_t j0;
+        if (!sq.next(hist, j0)) return false;
         const int s = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1u;
-        if (wait_or_abort(&kv_empty[s], ph ^ 1u, p.err, aborted)) {
-          uint8_t* kd = sStage + s * C::kStageBytes;
-          uint8_t* vd = kd + C::kTileBytes;
-          mbar_arrive_expect_tx(&kv_full[s], C::kStageBytes);
+        if (wait_or_abort(&empty[s], ph ^ 1u, p.err, aborted)) {
+          uint8_t* d = buf + s * C::kTileBytes;
+          mbar_arrive_expect_tx(&full[s], C::kTileBytes);
 #pragma unroll
           for (int sl = 0; sl < C::kSlabs; ++sl) {
 #pragma unroll
             for (int hf = 0; hf < BN / 64; ++hf) {
               const uint32_t off = sl * C::kKVSlab + hf * 64 * 128;
-              if (hist) {
-                tma_load_2d(kd + off, &ring_map, sl * 64, (int32_t)(krow0 + j0 + hf * 64), &kv_full[s]);
-                tma_load_2d(vd + off, &ring_map, sl * 64, (int32_t)(vrow0 + j0 + hf * 64), &kv_full[s]);
-              } else {
-                const int32_t z = (int32_t)((int64_t)b * p.n + j0 + hf * 64);
-                tma_load_3d(kd + off, &ck_map, sl * 64, h, z, &kv_full[s]);
-                tma_load_3d(vd + off, &cv_map, sl * 64, h, z, &kv_full[s]);
-              }
+              if (hist)
+                tma_load_2d(d + off, &ring_map, sl * 64, (int32_t)(row0 + j0 + hf * 64), &full[s]);
+              else
+                tma_load_3d(d + off, cmap, sl * 64, h, (int32_t)((int64_t)b * p.n + j0 + hf * 64),
+                            &full[s]);
             }
           }
         }
         ++it;
+        return true;
+      };
+      bool more_k = issue(seq, it_k, k_full, k_empty, sK, krow0, &ck_map);
+      while (true) {
+        if (more_k) more_k = issue(seq, it_k, k_full, k_empty, sK, krow0, &ck_map);
+        if (!issue(seq_v, it_v, v_full, v_empty, sV, vrow0, &cv_map)) break;
       }
       // every issued copy has landed before shared memory can go away
-      const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
       bool late = false;
-      for (uint32_t j = first; j < it; ++j)
-        wait_or_abort(&kv_full[j % STAGES], (j / STAGES) & 1u, p.err, late);
+      for (uint32_t j = it_k > (uint32_t)STAGES ? it_k - STAGES : 0u; j < it_k; ++j)
+        wait_or_abort(&k_full[j % STAGES], (j / STAGES) & 1u, p.err, late);
+      for (uint32_t j = it_v > (uint32_t)STAGES ? it_v - STAGES : 0u; j < it_v; ++j)
+        wait_or_abort(&v_full[j % STAGES], (j / STAGES) & 1u, p.err, late);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------- mma issuer
@@ -296,16 +311,18 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
       const uint32_t q_base = smem_u32(sQ);
       wait_or_abort(q_full, 0, p.err, aborted);
       auto issue_pv = [&](uint32_t jj) {
-        if (wait_or_abort(p_full, jj & 1u, p.err, aborted)) {
+        bool ok = wait_or_abort(p_full, jj & 1u, p.err, aborted);
+        ok = ok && wait_or_abort(&v_full[jj % STAGES], (jj / STAGES) & 1u, p.err, aborted);
+        if (ok) {
           tc_fence_after();
-          const uint32_t v_base = smem_u32(sStage + (jj % STAGES) * C::kStageBytes + C::kTileBytes);
+          const uint32_t v_base = smem_u32(sV + (jj % STAGES) * C::kTileBytes);
 #pragma unroll
           for (int kk = 0; kk < BN / 16; ++kk) {  // 16 keys = 8 packed P columns
             const uint64_t bd = smem_desc_sw128(v_base + kk * 2048, C::kKVSlab, 1024);
             umma_bf16_tmem_a(tO, tP + kk * 8, bd, idesc_pv, (jj > 0 || kk > 0) ? 1u : 0u);
           }
           umma_commit(pv_done);
-          umma_commit(&kv_empty[jj % STAGES]);
+          umma_commit(&v_empty[jj % STAGES]);
         }
       };
       uint32_t j = 0;
@@ -314,11 +331,11 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
       while (seq.next(hist, j0)) {
         const int s = j % STAGES;
         const int sb = j % SBUF;
-        bool ok = wait_or_abort(&kv_full[s], (j / STAGES) & 1u, p.err, aborted);
+        bool ok = wait_or_abort(&k_full[s], (j / STAGES) & 1u, p.err, aborted);
         ok = ok && wait_or_abort(&s_free[sb], ((j / SBUF) & 1u) ^ 1u, p.err, aborted);
         if (ok) {
           tc_fence_after();
-          const uint32_t k_base = smem_u32(sStage + s * C::kStageBytes);
+          const uint32_t k_base = smem_u32(sK + s * C::kTileBytes);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint64_t a = smem_desc_sw128(q_base + (kk >> 2) * C::kQSlab + (kk & 3) * 32, 16, 1024);
@@ -326,6 +343,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, STAGES, SPLIT, SBUF, CTAS>::kThre
             umma_bf16(tmem + sb * BN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
           }
           umma_commit(&s_full[sb]);
+          umma_commit(&k_empty[s]);  // the K tile is free once its QK^T has read it
         }
         if (j >= 1) issue_pv(j - 1);
         ++j;
