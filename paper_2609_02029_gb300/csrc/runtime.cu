@@ -410,6 +410,9 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
                   row0, (long long)t_rows, b, (long long)c->row_t(layer, b));
   if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
   if (n > (int64_t)65535 * 16) return fail(HWKV_EUNSUPPORTED, "chunk of %lld tokens too long", (long long)n);
+  // the prefill kernel walks positions and ring slots in 32-bit arithmetic
+  if (t_rows + n >= ((int64_t)1 << 30))
+    return fail(HWKV_EUNSUPPORTED, "prefill past 2^30 tokens of history");
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   PrefillParams p{};
   p.n_units = c->pol.n_kv_heads;
@@ -429,7 +432,10 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
   p.err = c->err();
   for (int h = 0; h < p.n_units; ++h) {
     const Unit& u = c->lay.units[(size_t)layer * p.n_units + h];
-    p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window, u.stride, u.sink};
+    if (u.cap >= ((int64_t)1 << 30)) return fail(HWKV_EUNSUPPORTED, "prefill into a ring of 2^30 slots or more");
+    // a window that reaches past every position the kernel can see is the full history
+    p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window >= ((int64_t)1 << 30) ? 0 : u.window,
+                         u.stride, u.sink};
   }
   // tensor maps of this call's q and chunk K/V: 3-D views {d, heads, batch * n}
   auto encode = get_encode();
