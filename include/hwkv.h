@@ -68,8 +68,8 @@ typedef enum {
  *     value of x / s (ties to even, saturating), value = code * s; a zero row
  *     stores s = 0. Effective precision (d + 4) / d bytes per element. Attention
  *     reads the dequantised rows (the paper: when the format changes execution,
- *     every compared output uses it). head_dim 128 or 256; hwkv_prefill is not
- *     built for it (rows enter through hwkv_append / the decode steps).
+ *     every compared output uses it), in prefill the chunk's own keys included
+ *     (they are read as the append stores them). head_dim 128 or 256.
  */
 #define HWKV_KV_BF16 0
 #define HWKV_KV_FP8_E4M3 1
@@ -150,7 +150,15 @@ HWKV_API hwkv_status hwkv_append(hwkv_cache* cache, int32_t layer, const void* k
  *   out: [batch, n, n_q_heads, head_dim] fp32, the per-head outputs
  *        concatenated in head order (pre-gate layout, Sec. 3.3).
  * Because attention runs before the write, a ring of capacity exactly W
- * serves chunks longer than W. Fails with HWKV_ECAPACITY as hwkv_append.
+ * serves chunks longer than W. Fails with HWKV_ECAPACITY as hwkv_append, and
+ * with HWKV_EUNSUPPORTED past 2^30 tokens of history or for chunks over
+ * 1,048,560 tokens.
+ * With HWKV_KV_FP8_E4M3 every key of the query's window is read as stored
+ * (code x scale), the chunk's own keys as the append will store them; the call
+ * allocates (stream-ordered) and frees a staging buffer of about
+ * 4 * head_dim bytes per ring slot of the layer and per chunk token and KV
+ * head (HWKV_ENOMEM if that fails). V rows are staged dequantized in fp16, so
+ * values past +-65504 saturate there.
  */
 HWKV_API hwkv_status hwkv_prefill(hwkv_cache* cache, int32_t layer, const void* q, const void* k,
                          const void* v, int64_t n, float scale, float* out, void* cuda_stream);

@@ -82,25 +82,11 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
         const uint2 v = *reinterpret_cast<const uint2*>(in[kv] + src);
         raw[0] = v.x; raw[1] = v.y;
       }
-      float amax = 0.f;
 #pragma unroll
-      for (int j = 0; j < PER; ++j) {
+      for (int j = 0; j < PER; ++j)
         x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
-        amax = fmaxf(amax, fabsf(x[j]));
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-      const float sc = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
       uint32_t w[PER / 4];
-#pragma unroll
-      for (int j = 0; j < PER; j += 4) {
-        uint32_t c01 = 0, c23 = 0;
-        if (amax > 0.f) {
-          c01 = f32x2_to_e4m3x2(__fdiv_rn(x[j], sc), __fdiv_rn(x[j + 1], sc));
-          c23 = f32x2_to_e4m3x2(__fdiv_rn(x[j + 2], sc), __fdiv_rn(x[j + 3], sc));
-        }
-        w[j / 4] = c01 | (c23 << 16);
-      }
+      const float sc = e4m3_quantize_row_warp<PER>(x, w);
       uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + rows[kv] * D + lane * PER;
       if constexpr (PER == 8)
         *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
@@ -109,6 +95,120 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
       if (lane == 0) p.scales[rows[kv]] = sc;
     }
   }
+}
+
+// Prefill staging for the 8-bit format, one warp per row. Ring rows: the slots of
+// (unit, batch row) below min(t0, cap); chunk rows: quantized as append_fp8_kernel
+// stores them (same helper). K rows become bf16 code values (E4M3 is exact in
+// bf16) plus their scales, applied to the logits in fp32; V rows become the
+// dequantized values code x scale in fp16 (11 significant bits; magnitudes past
+// the fp16 range saturate), so P stays a plain softmax weight.
+__device__ __forceinline__ void e4m3_words_to_16(const uint32_t* words, int nwords, bool as_f16,
+                                                 float sc, uint32_t* out) {
+  for (int i = 0; i < nwords; ++i) {
+    uint32_t lo, hi;
+    e4m3x4_to_f16x2(words[i], lo, hi);
+    const __half2 l2 = *reinterpret_cast<const __half2*>(&lo);
+    const __half2 h2 = *reinterpret_cast<const __half2*>(&hi);
+    if (as_f16) {
+      out[2 * i] = pack_f16_sat(__low2float(l2) * sc, __high2float(l2) * sc);
+      out[2 * i + 1] = pack_f16_sat(__low2float(h2) * sc, __high2float(h2) * sc);
+    } else {
+      out[2 * i] = pack_bf16(__low2float(l2), __high2float(l2));
+      out[2 * i + 1] = pack_bf16(__low2float(h2), __high2float(h2));
+    }
+  }
+}
+template <int D>
+__global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) {
+  constexpr int PER = D / 32;
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
+  const int64_t warp0 = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+  // ring rows: index over (unit, kv, batch row, slot < max cap)
+  int64_t max_cap = 0;
+  for (int h = 0; h < p.n_units; ++h) max_cap = p.u[h].cap > max_cap ? p.u[h].cap : max_cap;
+  const int64_t ring_items = (int64_t)p.n_units * 2 * p.batch * max_cap;
+  for (int64_t e = warp0; e < ring_items; e += warps) {
+    const int64_t slot = e % max_cap;
+    int64_t r = e / max_cap;
+    const int b = (int)(r % p.batch);
+    r /= p.batch;
+    const int kv = (int)(r % 2);
+    const int h = (int)(r / 2);
+    const Fp8StageUnit& u = p.u[h];
+    if (slot >= u.cap || slot >= p.t0) continue;
+    const int64_t src = (kv ? u.v_row0 : u.k_row0) + (int64_t)(p.row0 + b) * u.stride + slot;
+    const int64_t dst = (kv ? u.sv_row0 : u.sk_row0) + (int64_t)b * u.cap + slot;
+    const uint8_t* c = p.arena + src * D + lane * PER;
+    uint32_t words[PER / 4];
+    if constexpr (PER == 8) {
+      const uint2 w2 = *reinterpret_cast<const uint2*>(c);
+      words[0] = w2.x;
+      words[1] = w2.y;
+    } else {
+      words[0] = *reinterpret_cast<const uint32_t*>(c);
+    }
+    uint32_t out[PER / 2];
+    const float sc = p.arena_scales[src];
+    e4m3_words_to_16(words, PER / 4, kv == 1, sc, out);
+    __nv_bfloat16* o = p.ring_codes + dst * D + lane * PER;
+    if constexpr (PER == 8)
+      *reinterpret_cast<uint4*>(o) = make_uint4(out[0], out[1], out[2], out[3]);
+    else
+      *reinterpret_cast<uint2*>(o) = make_uint2(out[0], out[1]);
+    if (lane == 0 && kv == 0) p.ring_scales[dst] = sc;
+  }
+  // chunk rows: index over (batch row, token, unit)
+  const int64_t chunk_items = (int64_t)p.batch * p.n * p.n_units;
+  for (int64_t e = warp0; e < chunk_items; e += warps) {
+    const int h = (int)(e % p.n_units);
+    const int64_t r = e / p.n_units;  // b * n + i
+    const int64_t src = e * D + lane * PER;
+    const __nv_bfloat16* in[2] = {p.k, p.v};
+    __nv_bfloat16* outc[2] = {p.k_codes, p.v_codes};
+#pragma unroll
+    for (int kv = 0; kv < 2; ++kv) {
+      uint32_t raw[PER / 2];
+      if constexpr (PER == 8) {
+        const uint4 v = *reinterpret_cast<const uint4*>(in[kv] + src);
+        raw[0] = v.x; raw[1] = v.y; raw[2] = v.z; raw[3] = v.w;
+      } else {
+        const uint2 v = *reinterpret_cast<const uint2*>(in[kv] + src);
+        raw[0] = v.x; raw[1] = v.y;
+      }
+      float x[PER];
+#pragma unroll
+      for (int j = 0; j < PER; ++j)
+        x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
+      uint32_t w[PER / 4];
+      const float sc = e4m3_quantize_row_warp<PER>(x, w);
+      uint32_t out[PER / 2];
+      e4m3_words_to_16(w, PER / 4, kv == 1, sc, out);
+      __nv_bfloat16* o = outc[kv] + src;
+      if constexpr (PER == 8)
+        *reinterpret_cast<uint4*>(o) = make_uint4(out[0], out[1], out[2], out[3]);
+      else
+        *reinterpret_cast<uint2*>(o) = make_uint2(out[0], out[1]);
+      if (lane == 0 && kv == 0) p.k_scales[h * p.chunk_scale_stride + r] = sc;
+    }
+  }
+}
+
+cudaError_t launch_fp8_stage(const Fp8StageParams& p, int head_dim, cudaStream_t s) {
+  int64_t max_cap = 0;
+  for (int h = 0; h < p.n_units; ++h) max_cap = p.u[h].cap > max_cap ? p.u[h].cap : max_cap;
+  const int64_t rows = (int64_t)p.n_units * 2 * p.batch * max_cap + (int64_t)p.batch * p.n * p.n_units;
+  if (rows == 0) return cudaSuccess;
+  int64_t blocks = (rows + 7) / 8;  // 8 warps per block
+  const int64_t cap_blocks = 152 * 16;
+  if (blocks > cap_blocks) blocks = cap_blocks;
+  switch (head_dim) {
+    case 128: fp8_stage_kernel<128><<<(unsigned)blocks, 256, 0, s>>>(p); break;
+    case 256: fp8_stage_kernel<256><<<(unsigned)blocks, 256, 0, s>>>(p); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
 }
 
 cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s) {

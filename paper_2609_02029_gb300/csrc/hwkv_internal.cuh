@@ -135,19 +135,50 @@ struct PrefillParams {
   const __nv_bfloat16* v_arena;
   float* out;               // [batch][n][n_q_heads][D]
   int* err;
+  // 8-bit cache format: K tiles hold E4M3 code values (exact in bf16) and every key
+  // row an fp32 scale (ring scales indexed like the ring rows, chunk scales as
+  // [kv head][batch * n + 128]); V tiles hold the dequantized rows in fp16
+  const float* k_scale_ring;
+  const float* k_scale_chunk;
+  int64_t chunk_scale_stride;
   PrefillUnit u[kMaxKvHeads];
+};
+
+// Staging of an 8-bit cache for prefill: the visible ring rows of one layer and
+// the chunk's rows quantized exactly as the append stores them; K rows as bf16
+// code values plus row scales, V rows dequantized (code x scale) in fp16.
+struct Fp8StageUnit {
+  int64_t k_row0, v_row0, cap, stride, sink;  // arena rows
+  int64_t sk_row0, sv_row0;                   // staging rows (batch row b at + b * cap)
+};
+struct Fp8StageParams {
+  int32_t n_units, batch, row0;
+  int64_t t0, n;
+  const uint8_t* arena;           // E4M3 codes, one row of D bytes per arena row
+  const float* arena_scales;      // per arena row
+  __nv_bfloat16* ring_codes;      // staging rows x D (V rows: fp16 bits)
+  float* ring_scales;             // per staging row (K rows)
+  const __nv_bfloat16* k;         // chunk input [batch][n][n_units][D]
+  const __nv_bfloat16* v;
+  __nv_bfloat16* k_codes;         // chunk K code values, same layout
+  __nv_bfloat16* v_codes;         // chunk V rows dequantized (fp16 bits)
+  float* k_scales;                // [n_units][batch * n + 128]
+  int64_t chunk_scale_stride;
+  Fp8StageUnit u[kMaxKvHeads];
 };
 
 // launchers (defined in the kernel translation units); return cudaGetLastError()
 cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s);
+cudaError_t launch_fp8_stage(const Fp8StageParams& p, int head_dim, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& k_map,
                           const CUtensorMap& v_map, int head_dim, int grid, cudaStream_t s,
                           bool fp8 = false);
 cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cudaStream_t s);
 cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s);
+// fp8: K/V tiles are staged 8-bit rows (bf16 code values) with row scales in p
 cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtensorMap& q_map,
                               const CUtensorMap& ck_map, const CUtensorMap& cv_map,
-                              const CUtensorMap& ring_map, cudaStream_t s);
+                              const CUtensorMap& ring_map, cudaStream_t s, bool fp8 = false);
 int decode_smem_bytes(int head_dim);
 cudaError_t decode_prepare_device();  // one-time kernel attributes on the current device
 
@@ -351,9 +382,39 @@ __device__ __forceinline__ uint32_t f32x2_to_e4m3x2(float lo, float hi) {
   return d;
 }
 
+// One row quantized to the 8-bit format by a warp, each lane holding PER of its
+// values: amax = max |x| over the row; s = amax / 448 (IEEE division); code =
+// E4M3 of x / s (IEEE division, round to nearest even, saturating); amax = 0 gives
+// s = 0 and zero codes. Returns s; w[i] packs the codes of x[4i .. 4i + 3].
+template <int PER>
+__device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], uint32_t (&w)[PER / 4]) {
+  float amax = 0.f;
+#pragma unroll
+  for (int j = 0; j < PER; ++j) amax = fmaxf(amax, fabsf(x[j]));
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+  const float sc = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
+#pragma unroll
+  for (int j = 0; j < PER; j += 4) {
+    uint32_t c01 = 0, c23 = 0;
+    if (amax > 0.f) {
+      c01 = f32x2_to_e4m3x2(__fdiv_rn(x[j], sc), __fdiv_rn(x[j + 1], sc));
+      c23 = f32x2_to_e4m3x2(__fdiv_rn(x[j + 2], sc), __fdiv_rn(x[j + 3], sc));
+    }
+    w[j / 4] = c01 | (c23 << 16);
+  }
+  return sc;
+}
+
 __device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
   uint32_t d;
   asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+// as pack_f16, magnitudes past the fp16 range saturating to +-65504
+__device__ __forceinline__ uint32_t pack_f16_sat(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
   return d;
 }
 
@@ -489,6 +550,11 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
          ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+// The same with fp16 A and B (both operands of one mma share the type).
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N, bool b_mn_major) {
+  return (1u << 4) | ((b_mn_major ? 1u : 0u) << 16) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(M >> 4) << 24);
 }
 
 #endif  // __CUDACC__

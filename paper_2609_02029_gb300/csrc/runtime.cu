@@ -401,7 +401,6 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
   if (n < 0) return fail(HWKV_EINVAL, "n must be >= 0");
   if (n == 0) return ok();
   if (!q || !k || !v || !out) return fail(HWKV_EINVAL, "q/k/v/out is NULL");
-  if (c->fp8()) return fail(HWKV_EUNSUPPORTED, "prefill is not built for the 8-bit cache format");
   if ((st = check_room(c, layer, row0, n_rows, n)) != HWKV_OK) return st;
   const int64_t t_rows = c->row_t(layer, row0);
   for (int b = row0 + 1; b < row0 + n_rows; ++b)
@@ -452,27 +451,99 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(HWKV_EINVAL, "q tensor map rejected (%d): q must be 16-byte aligned", (int)r);
   }
-  {
-    const cuuint64_t dim[3] = {(cuuint64_t)d, (cuuint64_t)c->pol.n_kv_heads,
-                               (cuuint64_t)n_rows * (cuuint64_t)n};
-    const cuuint64_t str[2] = {(cuuint64_t)d * 2, (cuuint64_t)c->pol.n_kv_heads * d * 2};
-    const cuuint32_t box[3] = {64, 1, 64};
-    CUresult r = encode(&ck_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(k), dim,
-                        str, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r == CUDA_SUCCESS)
-      r = encode(&cv_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(v), dim, str,
-                 box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return fail(HWKV_EINVAL, "k/v tensor map rejected (%d): k/v must be 16-byte aligned", (int)r);
-  }
   if ((int64_t)n_rows * n + 128 >= (int64_t)INT32_MAX)
     return fail(HWKV_EUNSUPPORTED, "batch x chunk exceeds the TMA coordinate range");
-  cudaError_t e = launch_prefill_tc(p, d, q_map, ck_map, cv_map, c->kv_map, s);
-  if (e != cudaSuccess) return fail(HWKV_ECUDA, "prefill launch: %s", cudaGetErrorString(e));
+  const int H = c->pol.n_kv_heads;
+  auto encode_chunk = [&](CUtensorMap* m, const void* base) -> CUresult {
+    const cuuint64_t dim[3] = {(cuuint64_t)d, (cuuint64_t)H, (cuuint64_t)n_rows * (cuuint64_t)n};
+    const cuuint64_t str[2] = {(cuuint64_t)d * 2, (cuuint64_t)H * d * 2};
+    const cuuint32_t box[3] = {64, 1, 64};
+    return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dim, str, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  };
+  cudaError_t e = cudaSuccess;
+  if (!c->fp8()) {
+    CUresult r = encode_chunk(&ck_map, k);
+    if (r == CUDA_SUCCESS) r = encode_chunk(&cv_map, v);
+    if (r != CUDA_SUCCESS) return fail(HWKV_EINVAL, "k/v tensor map rejected (%d): k/v must be 16-byte aligned", (int)r);
+    e = launch_prefill_tc(p, d, q_map, ck_map, cv_map, c->kv_map, s);
+    if (e != cudaSuccess) return fail(HWKV_ECUDA, "prefill launch: %s", cudaGetErrorString(e));
+  } else {
+    // 8-bit cache: attention reads every key as stored (code x row scale), the
+    // chunk's own rows included. The visible ring rows are staged and the chunk
+    // quantized as the append will store it: K as bf16 code values (exact) whose
+    // scales the kernel applies to the logits in fp32, V dequantized in fp16.
+    if (!c->pol.head_dim || (d != 128 && d != 256))
+      return fail(HWKV_EUNSUPPORTED, "8-bit prefill needs head_dim 128 or 256");
+    Fp8StageParams sp{};
+    sp.n_units = H;
+    sp.batch = n_rows;
+    sp.row0 = row0;
+    sp.t0 = t_rows;
+    sp.n = n;
+    sp.arena = reinterpret_cast<const uint8_t*>(c->k_base());
+    sp.arena_scales = c->scales();
+    sp.k = static_cast<const __nv_bfloat16*>(k);
+    sp.v = static_cast<const __nv_bfloat16*>(v);
+    int64_t rows = 0;
+    for (int h = 0; h < H; ++h) {
+      const Unit& u = c->lay.units[(size_t)layer * H + h];
+      sp.u[h] = Fp8StageUnit{u.k_row0, u.v_row0, u.cap, u.stride, u.sink, rows, rows + (int64_t)n_rows * u.cap};
+      rows += 2 * (int64_t)n_rows * u.cap;
+    }
+    const int64_t cstride = (int64_t)n_rows * n + 128;
+    const size_t ring_code_bytes = align_up((size_t)rows * d * 2, 1024);
+    const size_t ring_scale_bytes = align_up((size_t)(rows + 128) * 4, 1024);
+    const size_t chunk_code_bytes = align_up((size_t)n_rows * n * H * d * 2, 1024);
+    const size_t chunk_scale_bytes = align_up((size_t)H * cstride * 4, 1024);
+    const size_t total = ring_code_bytes + ring_scale_bytes + 2 * chunk_code_bytes + chunk_scale_bytes;
+    uint8_t* buf = nullptr;
+    e = cudaMallocAsync(reinterpret_cast<void**>(&buf), total, s);
+    if (e != cudaSuccess) return fail(HWKV_ENOMEM, "8-bit prefill staging (%zu bytes): %s", total, cudaGetErrorString(e));
+    // zeros where nothing is staged: tiles read past the held rows (masked there,
+    // but a weight of 0 times a non-finite value would still poison the sum)
+    e = cudaMemsetAsync(buf, 0, total, s);
+    sp.ring_codes = reinterpret_cast<__nv_bfloat16*>(buf);
+    sp.ring_scales = reinterpret_cast<float*>(buf + ring_code_bytes);
+    sp.k_codes = reinterpret_cast<__nv_bfloat16*>(buf + ring_code_bytes + ring_scale_bytes);
+    sp.v_codes = reinterpret_cast<__nv_bfloat16*>(buf + ring_code_bytes + ring_scale_bytes + chunk_code_bytes);
+    sp.k_scales = reinterpret_cast<float*>(buf + ring_code_bytes + ring_scale_bytes + 2 * chunk_code_bytes);
+    sp.chunk_scale_stride = cstride;
+    if (e == cudaSuccess) e = launch_fp8_stage(sp, d, s);
+    CUtensorMap ring_map;
+    CUresult r = CUDA_SUCCESS;
+    if (e == cudaSuccess) {
+      const cuuint64_t gdim[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+      const cuuint64_t gstride[1] = {(cuuint64_t)d * 2};
+      const cuuint32_t box[2] = {64u, (cuuint32_t)kStageTokens};
+      const cuuint32_t es2[2] = {1, 1};
+      r = encode(&ring_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, sp.ring_codes, gdim, gstride, box, es2,
+                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r == CUDA_SUCCESS) r = encode_chunk(&ck_map, sp.k_codes);
+      if (r == CUDA_SUCCESS) r = encode_chunk(&cv_map, sp.v_codes);
+    }
+    if (e == cudaSuccess && r == CUDA_SUCCESS) {
+      for (int h = 0; h < H; ++h) {
+        p.u[h].k_row0 = sp.u[h].sk_row0;
+        p.u[h].v_row0 = sp.u[h].sv_row0;
+        p.u[h].stride = sp.u[h].cap;
+      }
+      p.row0 = 0;
+      p.k_scale_ring = sp.ring_scales;
+      p.k_scale_chunk = sp.k_scales;
+      p.chunk_scale_stride = cstride;
+      e = launch_prefill_tc(p, d, q_map, ck_map, cv_map, ring_map, s, true);
+    }
+    const cudaError_t ef = cudaFreeAsync(buf, s);
+    if (r != CUDA_SUCCESS) return fail(HWKV_ECUDA, "8-bit prefill tensor maps rejected (%d)", (int)r);
+    if (e != cudaSuccess) return fail(HWKV_ECUDA, "8-bit prefill launch: %s", cudaGetErrorString(e));
+    if (ef != cudaSuccess) return fail(HWKV_ECUDA, "8-bit prefill staging free: %s", cudaGetErrorString(ef));
+  }
   // attend first, then write the chunk's retained tokens (stream order)
   const AppendParams ap = append_params(c, layer, row0, n_rows, k, v, n);
-  e = launch_append(ap, false, s);
+  e = launch_append(ap, c->fp8(), s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "append launch: %s", cudaGetErrorString(e));
   for (int b = row0; b < row0 + n_rows; ++b) c->row_t(layer, b) += n;
   return ok();

@@ -1,9 +1,10 @@
 """The 8-bit cache format (E4M3 codes + one fp32 scale per stored row) through
 the C ABI, against the oracle's encoding written from the format definition:
 ring codes and scales bit-exact (the quantisation decisions are taken in fp32
-on both sides), decode outputs within the attention tolerance of the oracle's
-attention over the dequantised rows (Sec. 3.1: with a format that changes
-execution, the compared outputs all use it)."""
+on both sides), decode and prefill outputs within the attention tolerance of the
+oracle's attention over the dequantised rows (Sec. 3.1: with a format that
+changes execution, the compared outputs all use it; a prefill chunk's own keys
+are read as stored too)."""
 import numpy as np
 import pytest
 
@@ -195,19 +196,71 @@ def test_fp8_larger_sampled():
         r.close()
 
 
-def test_fp8_unsupported_paths():
-    import torch
+def test_fp8_unsupported_head_dim():
     with pytest.raises(hwkv.HwkvError) as e:
         pol = hwkv.make_policy(1, 1, 1, 64, 1, 100, [0], kv_format=FP8)
         hwkv.hwkv_required_bytes(pol)
     assert e.value.status == hwkv.HWKV_EUNSUPPORTED
-    r = Run8(1, 1, 2, 1, 128, 100, [0], seed=1)
+
+
+def prefill_chunk(r, layer, n, row0=None, n_rows=None):
+    """Prefill n tokens of the generator's q/k/v into rows [row0, row0 + n_rows)."""
+    import torch
+    row0 = 0 if row0 is None else row0
+    n_rows = r.B if n_rows is None else n_rows
+    t0 = hwkv.hwkv_row_len(r.cache, layer, row0)
+    def gen(tensor, heads):
+        full = r.gen(tensor, layer, t0, n, heads)
+        return full[row0:row0 + n_rows].contiguous()
+    q, k, v = gen(hwkv_gen.Q, r.Hq), gen(hwkv_gen.K, r.Hkv), gen(hwkv_gen.V, r.Hkv)
+    out = torch.empty((n_rows, n, r.Hq, r.d), dtype=torch.float32, device="cuda")
+    if n_rows == r.B:
+        hwkv.hwkv_prefill(r.cache, layer, q, k, v, n, r.scale, out, r.stream)
+    else:
+        hwkv.hwkv_prefill_rows(r.cache, layer, row0, n_rows, q, k, v, n, r.scale, out, r.stream)
+    return t0, out.cpu().numpy()
+
+
+def check_prefill(r, layer, t0, n, got, row0=0, stride=13):
+    pos = sorted(set(range(t0, t0 + n, stride)) | {t0, t0 + n - 1})
+    for bi in range(got.shape[0]):
+        for h in range(r.Hkv):
+            for p in pos:
+                want = r.oracle_unit(layer, row0 + bi, h, p)
+                assert_close(got[bi, p - t0, h * r.G:(h + 1) * r.G], want,
+                             "fp8 prefill b=%d h=%d p=%d" % (row0 + bi, h, p))
+
+
+@pytest.mark.parametrize("d", [128, 256])
+def test_fp8_prefill_parity_and_rings(d):
+    # a full head and a 100-token window; chunks from an empty cache, past the
+    # window (the ring wraps inside the call) and after appended history
+    r = Run8(1, 2, 8, 2, d, 1400, [0, 100], seed=23)
     try:
-        q = torch.zeros((1, 4, 2, 128), dtype=torch.bfloat16, device="cuda")
-        kv = torch.zeros((1, 4, 1, 128), dtype=torch.bfloat16, device="cuda")
-        out = torch.empty((1, 4, 2, 128), dtype=torch.float32, device="cuda")
-        with pytest.raises(hwkv.HwkvError) as e:
-            hwkv.hwkv_prefill(r.cache, 0, q, kv, kv, 4, r.scale, out, r.stream)
-        assert e.value.status == hwkv.HWKV_EUNSUPPORTED
+        for n in (70, 333):
+            t0, got = prefill_chunk(r, 0, n)
+            check_prefill(r, 0, t0, n, got)
+            r.check_rings(0)
+        r.fill(0, 41)
+        t0, got = prefill_chunk(r, 0, 150)
+        check_prefill(r, 0, t0, 150, got)
+        r.check_rings(0)
+        t = hwkv.hwkv_seq_len(r.cache, 0)
+        out = r.step(0, fused=True)
+        assert_close(out.cpu().numpy(), r.oracle_step(0, t), "fp8 decode after prefill d=%d" % d)
+        hwkv.hwkv_sync_check(r.cache)
+    finally:
+        r.close()
+
+
+def test_fp8_prefill_rows_ragged():
+    # rows of one cache at different lengths: a row range prefilled on its own
+    r = Run8(1, 3, 8, 2, 128, 900, [0, 64], seed=29)
+    try:
+        t0, got = prefill_chunk(r, 0, 90)
+        t0, got = prefill_chunk(r, 0, 130, row0=1, n_rows=2)
+        assert [hwkv.hwkv_row_len(r.cache, 0, b) for b in range(3)] == [90, 220, 220]
+        check_prefill(r, 0, t0, 130, got, row0=1, stride=11)
+        hwkv.hwkv_sync_check(r.cache)
     finally:
         r.close()

@@ -3,7 +3,7 @@ StreamingLLM control: S sink tokens plus a W-token window) through the C ABI:
 prefill chunks that start below, inside and past the sink region, appends that
 wrap the window region, decode (plain, fused, captured graph), ring contents
 bit-exact against the oracle's ring, residency by the retained-count closed
-form, and 8-bit rings of sink heads."""
+form, and 8-bit rings and prefill of sink heads."""
 import numpy as np
 import pytest
 
@@ -50,6 +50,26 @@ class RunS:
         np.testing.assert_allclose(sp, 1.0, atol=1e-12)
         return O
 
+    def oracle_rows_fp8(self, b, qh, positions):
+        """8-bit format: attention (the plain definition over J) over the rows as
+        stored, quantized and dequantized, every key of J included."""
+        h = qh // self.G
+        W, S = self.windows[h], self.sinks[h]
+        out = np.zeros((len(positions), self.d))
+        for i, p in enumerate(positions):
+            J = oracle.sink_positions(p, W, S)
+            rows = {}
+            for tensor in (hwkv_gen.K, hwkv_gen.V):
+                X = np.stack([hwkv_gen.fill_host_sub(self.g, tensor, 0, b, int(k), 1, h, 1, self.d)[0, 0]
+                              for k in J])
+                codes, scales = oracle.quantize_rows_e4m3(X)
+                rows[tensor] = oracle.dequantize_rows_e4m3(codes, scales)
+            qb = hwkv_gen.fill_host_sub(self.g, hwkv_gen.Q, 0, b, p, 1, qh, 1, self.d)[0, 0]
+            q = (qb.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+            out[i], pi = oracle.attend(q, rows[hwkv_gen.K], rows[hwkv_gen.V], self.scale)
+            np.testing.assert_allclose(pi.sum(), 1.0, atol=1e-12)
+        return out
+
     def prefill(self, n, sample=17):
         t0 = hwkv.hwkv_seq_len(self.cache, 0)
         q, k, v = self.gen(hwkv_gen.Q, t0, n, self.Hq), self.gen(hwkv_gen.K, t0, n, self.Hkv), \
@@ -61,7 +81,9 @@ class RunS:
         pos = sorted(set(list(range(t0, t0 + n, sample)) + [t0, t0 + n - 1]))
         for b in range(self.B):
             for qh in range(0, self.Hq, 3):
-                assert_close(got[b, [p - t0 for p in pos], qh], self.oracle_rows(b, qh, pos),
+                want = (self.oracle_rows(b, qh, pos) if self.fmt == hwkv.HWKV_KV_BF16 else
+                        self.oracle_rows_fp8(b, qh, pos))
+                assert_close(got[b, [p - t0 for p in pos], qh], want,
                              "prefill t0=%d b=%d qh=%d" % (t0, b, qh))
 
     def append(self, n):
@@ -183,6 +205,20 @@ def test_sink_rings_in_8_bits():
         for _ in range(2):
             t = hwkv.hwkv_seq_len(r.cache, 0)
             out = torch_step_fp8(r, t)
+        hwkv.hwkv_sync_check(r.cache)
+        r.check_rings()
+        r.check_residency()
+    finally:
+        r.close()
+
+
+def test_sink_prefill_8_bits():
+    r = RunS(windows=[48, 0], sinks=[5, 0], head_dim=128, max_ctx=700, seed=12,
+             kv_format=hwkv.HWKV_KV_FP8_E4M3)
+    try:
+        r.prefill(3, sample=1)   # inside the sink region
+        r.prefill(100)           # through the sinks, wraps the window region
+        r.prefill(150)
         hwkv.hwkv_sync_check(r.cache)
         r.check_rings()
         r.check_residency()
