@@ -264,3 +264,46 @@ def test_fp8_prefill_rows_ragged():
         hwkv.hwkv_sync_check(r.cache)
     finally:
         r.close()
+
+
+def test_prefill64k_fp8_sampled():
+    """The bench's 8-bit prefill (prefill64k: 8 chunks of 8,192 tokens, B2, 32q/8kv, d128,
+    windows drawn per KV head) on sampled rows of the first and the last chunk, for one
+    full-history and one windowed KV head per batch row."""
+    from hwkv_gen import workloads
+    wl = workloads.make("prefill64k")
+    r = Run8(wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.max_ctx,
+             wl.windows, seed=wl.seed, per_head_scale=wl.per_head_scale)
+    rng = np.random.default_rng(5)
+    try:
+        n = wl.chunk
+        kept = {}
+        for c in range(wl.prompt // n):
+            t0, got = prefill_chunk(r, 0, n)
+            if c in (0, wl.prompt // n - 1):
+                kept[c] = (t0, got)
+        hwkv.hwkv_sync_check(r.cache)
+        full = [h for h in range(r.Hkv) if r.window(0, h) == 0 or r.window(0, h) >= r.max_ctx]
+        win = [h for h in range(r.Hkv) if h not in full]
+        heads = ([full[0]] if full else []) + ([win[0]] if win else [])
+        for c, (t0, got) in kept.items():
+            rows = sorted({0, n - 1} | set(rng.integers(0, n, size=6).tolist()))
+            pos = [t0 + i for i in rows]
+            for b in range(r.B):
+                for h in heads:
+                    T = pos[-1] + 1
+                    K = hwkv_gen.fill_host_sub(r.g, hwkv_gen.K, 0, b, 0, T, h, 1, r.d)[:, 0]
+                    V = hwkv_gen.fill_host_sub(r.g, hwkv_gen.V, 0, b, 0, T, h, 1, r.d)[:, 0]
+                    Kc, Ks = oracle.quantize_rows_e4m3(K)
+                    Vc, Vs = oracle.quantize_rows_e4m3(V)
+                    W = r.window(0, h)
+                    W = 0 if W >= r.max_ctx else W
+                    for qg in range(r.G):
+                        qh = h * r.G + qg
+                        Q = np.stack([hwkv_gen.fill_host_sub(r.g, hwkv_gen.Q, 0, b, p, 1, qh, 1, r.d)[0, 0]
+                                      for p in pos])
+                        O, sp = oracle.window_attention_fp8(Q, pos, Kc, Ks, Vc, Vs, W, r.scale)
+                        np.testing.assert_allclose(sp, 1.0, atol=1e-12)
+                        assert_close(got[b, rows, qh], O, "fp8 prefill64k chunk %d b%d q%d" % (c, b, qh))
+    finally:
+        r.close()
