@@ -769,7 +769,7 @@ def main():
             line["prefill"]["fp8_kv"] = {
                 "tflops": pre8["tflops"], "ms": pre8["ms"], "tokens_per_s": pre8["tokens_per_s"],
                 "note": "same prompt with the cache in E4M3 codes + row scales; each call stages "
-                        "the visible rows (K codes, V dequantized to fp16) and appends in 8 bits"}
+                        "q and the held/new K/V rows dequantized in fp16, then appends in 8 bits"}
     if cal is not None:
         line["seqcalib"] = cal
     if cb is not None:

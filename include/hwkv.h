@@ -155,10 +155,10 @@ HWKV_API hwkv_status hwkv_append(hwkv_cache* cache, int32_t layer, const void* k
  * 1,048,560 tokens.
  * With HWKV_KV_FP8_E4M3 every key of the query's window is read as stored
  * (code x scale), the chunk's own keys as the append will store them; the call
- * allocates (stream-ordered) and frees a staging buffer of about
- * 4 * head_dim bytes per ring slot of the layer and per chunk token and KV
- * head (HWKV_ENOMEM if that fails). V rows are staged dequantized in fp16, so
- * values past +-65504 saturate there.
+ * allocates (stream-ordered) and frees a staging buffer of 2 * head_dim bytes
+ * per held ring slot of the layer (K and V) and per chunk token and head (q, K,
+ * V) (HWKV_ENOMEM if that fails): q and the dequantized K/V rows go through the
+ * tensor cores in fp16, so magnitudes past +-65504 saturate there.
  */
 HWKV_API hwkv_status hwkv_prefill(hwkv_cache* cache, int32_t layer, const void* q, const void* k,
                          const void* v, int64_t n, float scale, float* out, void* cuda_stream);

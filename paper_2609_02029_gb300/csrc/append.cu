@@ -97,108 +97,119 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   }
 }
 
-// Prefill staging for the 8-bit format, one warp per row. Ring rows: the slots of
-// (unit, batch row) below min(t0, cap); chunk rows: quantized as append_fp8_kernel
-// stores them (same helper). K rows become bf16 code values (E4M3 is exact in
-// bf16) plus their scales, applied to the logits in fp32; V rows become the
-// dequantized values code x scale in fp16 (11 significant bits; magnitudes past
-// the fp16 range saturate), so P stays a plain softmax weight.
-__device__ __forceinline__ void e4m3_words_to_16(const uint32_t* words, int nwords, bool as_f16,
-                                                 float sc, uint32_t* out) {
+// Prefill staging for the 8-bit format, one warp per row, everything in fp16 for
+// an fp16 tensor-core pass. Ring rows: the held slots of (unit, batch row), below
+// min(t0, cap), dequantized (code x scale), and zeros for the next 128 slots, which
+// a key tile may read past them. Chunk K/V rows: quantized as append_fp8_kernel
+// stores them (same helper), then dequantized. q rows: converted. fp16 keeps 11
+// significant bits; magnitudes past its range saturate to +-65504.
+__device__ __forceinline__ void e4m3_words_to_f16(const uint32_t* words, int nwords, float sc,
+                                                  uint32_t* out) {
   for (int i = 0; i < nwords; ++i) {
     uint32_t lo, hi;
     e4m3x4_to_f16x2(words[i], lo, hi);
     const __half2 l2 = *reinterpret_cast<const __half2*>(&lo);
     const __half2 h2 = *reinterpret_cast<const __half2*>(&hi);
-    if (as_f16) {
-      out[2 * i] = pack_f16_sat(__low2float(l2) * sc, __high2float(l2) * sc);
-      out[2 * i + 1] = pack_f16_sat(__low2float(h2) * sc, __high2float(h2) * sc);
-    } else {
-      out[2 * i] = pack_bf16(__low2float(l2), __high2float(l2));
-      out[2 * i + 1] = pack_bf16(__low2float(h2), __high2float(h2));
-    }
+    out[2 * i] = pack_f16_sat(__low2float(l2) * sc, __high2float(l2) * sc);
+    out[2 * i + 1] = pack_f16_sat(__low2float(h2) * sc, __high2float(h2) * sc);
   }
 }
+template <int PER>
+__device__ __forceinline__ void store_row16(uint16_t* dst, const uint32_t (&w)[PER / 2]) {
+  if constexpr (PER == 8)
+    *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+  else
+    *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
+}
+template <int PER>
+__device__ __forceinline__ void load_row_bf16(const __nv_bfloat16* src, float (&x)[PER]) {
+  uint32_t raw[PER / 2];
+  if constexpr (PER == 8) {
+    const uint4 v = *reinterpret_cast<const uint4*>(src);
+    raw[0] = v.x; raw[1] = v.y; raw[2] = v.z; raw[3] = v.w;
+  } else {
+    const uint2 v = *reinterpret_cast<const uint2*>(src);
+    raw[0] = v.x; raw[1] = v.y;
+  }
+#pragma unroll
+  for (int j = 0; j < PER; ++j)
+    x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
+}
+
 template <int D>
 __global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) {
   constexpr int PER = D / 32;
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
   const int64_t warp0 = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
-  // ring rows: index over (unit, kv, batch row, slot < max cap)
+  // ring rows: index over (unit, kv, batch row, slot < span)
   int64_t max_cap = 0;
   for (int h = 0; h < p.n_units; ++h) max_cap = p.u[h].cap > max_cap ? p.u[h].cap : max_cap;
-  const int64_t ring_items = (int64_t)p.n_units * 2 * p.batch * max_cap;
+  const int64_t span = min(max_cap, p.t0 + 128);
+  const int64_t ring_items = (int64_t)p.n_units * 2 * p.batch * span;
   for (int64_t e = warp0; e < ring_items; e += warps) {
-    const int64_t slot = e % max_cap;
-    int64_t r = e / max_cap;
+    const int64_t slot = e % span;
+    int64_t r = e / span;
     const int b = (int)(r % p.batch);
     r /= p.batch;
     const int kv = (int)(r % 2);
     const int h = (int)(r / 2);
     const Fp8StageUnit& u = p.u[h];
-    if (slot >= u.cap || slot >= p.t0) continue;
+    if (slot >= u.cap) continue;
     const int64_t src = (kv ? u.v_row0 : u.k_row0) + (int64_t)(p.row0 + b) * u.stride + slot;
     const int64_t dst = (kv ? u.sv_row0 : u.sk_row0) + (int64_t)b * u.cap + slot;
-    const uint8_t* c = p.arena + src * D + lane * PER;
-    uint32_t words[PER / 4];
-    if constexpr (PER == 8) {
-      const uint2 w2 = *reinterpret_cast<const uint2*>(c);
-      words[0] = w2.x;
-      words[1] = w2.y;
-    } else {
-      words[0] = *reinterpret_cast<const uint32_t*>(c);
-    }
     uint32_t out[PER / 2];
-    const float sc = p.arena_scales[src];
-    e4m3_words_to_16(words, PER / 4, kv == 1, sc, out);
-    __nv_bfloat16* o = p.ring_codes + dst * D + lane * PER;
-    if constexpr (PER == 8)
-      *reinterpret_cast<uint4*>(o) = make_uint4(out[0], out[1], out[2], out[3]);
-    else
-      *reinterpret_cast<uint2*>(o) = make_uint2(out[0], out[1]);
-    if (lane == 0 && kv == 0) p.ring_scales[dst] = sc;
+    if (slot >= p.t0) {  // not held
+#pragma unroll
+      for (int i = 0; i < PER / 2; ++i) out[i] = 0u;
+    } else {
+      const uint8_t* c = p.arena + src * D + lane * PER;
+      uint32_t words[PER / 4];
+      if constexpr (PER == 8) {
+        const uint2 w2 = *reinterpret_cast<const uint2*>(c);
+        words[0] = w2.x;
+        words[1] = w2.y;
+      } else {
+        words[0] = *reinterpret_cast<const uint32_t*>(c);
+      }
+      e4m3_words_to_f16(words, PER / 4, p.arena_scales[src], out);
+    }
+    store_row16<PER>(p.ring + dst * D + lane * PER, out);
   }
-  // chunk rows: index over (batch row, token, unit)
+  // chunk rows: index over (batch row, token, KV head)
   const int64_t chunk_items = (int64_t)p.batch * p.n * p.n_units;
   for (int64_t e = warp0; e < chunk_items; e += warps) {
-    const int h = (int)(e % p.n_units);
-    const int64_t r = e / p.n_units;  // b * n + i
-    const int64_t src = e * D + lane * PER;
-    const __nv_bfloat16* in[2] = {p.k, p.v};
-    __nv_bfloat16* outc[2] = {p.k_codes, p.v_codes};
+    const int64_t off = e * D + lane * PER;
 #pragma unroll
     for (int kv = 0; kv < 2; ++kv) {
-      uint32_t raw[PER / 2];
-      if constexpr (PER == 8) {
-        const uint4 v = *reinterpret_cast<const uint4*>(in[kv] + src);
-        raw[0] = v.x; raw[1] = v.y; raw[2] = v.z; raw[3] = v.w;
-      } else {
-        const uint2 v = *reinterpret_cast<const uint2*>(in[kv] + src);
-        raw[0] = v.x; raw[1] = v.y;
-      }
       float x[PER];
-#pragma unroll
-      for (int j = 0; j < PER; ++j)
-        x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
+      load_row_bf16<PER>((kv ? p.v : p.k) + off, x);
       uint32_t w[PER / 4];
       const float sc = e4m3_quantize_row_warp<PER>(x, w);
       uint32_t out[PER / 2];
-      e4m3_words_to_16(w, PER / 4, kv == 1, sc, out);
-      __nv_bfloat16* o = outc[kv] + src;
-      if constexpr (PER == 8)
-        *reinterpret_cast<uint4*>(o) = make_uint4(out[0], out[1], out[2], out[3]);
-      else
-        *reinterpret_cast<uint2*>(o) = make_uint2(out[0], out[1]);
-      if (lane == 0 && kv == 0) p.k_scales[h * p.chunk_scale_stride + r] = sc;
+      e4m3_words_to_f16(w, PER / 4, sc, out);
+      store_row16<PER>((kv ? p.v16 : p.k16) + off, out);
     }
+  }
+  // q rows: index over (batch row, token, query head)
+  const int64_t q_items = (int64_t)p.batch * p.n * p.n_q_heads;
+  for (int64_t e = warp0; e < q_items; e += warps) {
+    const int64_t off = e * D + lane * PER;
+    float x[PER];
+    load_row_bf16<PER>(p.q + off, x);
+    uint32_t out[PER / 2];
+#pragma unroll
+    for (int i = 0; i < PER / 2; ++i) out[i] = pack_f16_sat(x[2 * i], x[2 * i + 1]);
+    store_row16<PER>(p.q16 + off, out);
   }
 }
 
 cudaError_t launch_fp8_stage(const Fp8StageParams& p, int head_dim, cudaStream_t s) {
   int64_t max_cap = 0;
   for (int h = 0; h < p.n_units; ++h) max_cap = p.u[h].cap > max_cap ? p.u[h].cap : max_cap;
-  const int64_t rows = (int64_t)p.n_units * 2 * p.batch * max_cap + (int64_t)p.batch * p.n * p.n_units;
+  const int64_t span = min(max_cap, p.t0 + 128);
+  const int64_t rows = (int64_t)p.n_units * 2 * p.batch * span +
+                       (int64_t)p.batch * p.n * (p.n_units + p.n_q_heads);
   if (rows == 0) return cudaSuccess;
   int64_t blocks = (rows + 7) / 8;  // 8 warps per block
   const int64_t cap_blocks = 152 * 16;

@@ -135,35 +135,28 @@ struct PrefillParams {
   const __nv_bfloat16* v_arena;
   float* out;               // [batch][n][n_q_heads][D]
   int* err;
-  // 8-bit cache format: K tiles hold E4M3 code values (exact in bf16) and every key
-  // row an fp32 scale (ring scales indexed like the ring rows, chunk scales as
-  // [kv head][batch * n + 128]); V tiles hold the dequantized rows in fp16
-  const float* k_scale_ring;
-  const float* k_scale_chunk;
-  int64_t chunk_scale_stride;
   PrefillUnit u[kMaxKvHeads];
 };
 
-// Staging of an 8-bit cache for prefill: the visible ring rows of one layer and
-// the chunk's rows quantized exactly as the append stores them; K rows as bf16
-// code values plus row scales, V rows dequantized (code x scale) in fp16.
+// Staging of an 8-bit cache for prefill, everything in fp16 for an fp16 tensor-core
+// pass: the visible ring rows of one layer dequantized (code x scale), the chunk's
+// K/V rows quantized exactly as the append stores them and dequantized, and q.
 struct Fp8StageUnit {
   int64_t k_row0, v_row0, cap, stride, sink;  // arena rows
   int64_t sk_row0, sv_row0;                   // staging rows (batch row b at + b * cap)
 };
 struct Fp8StageParams {
-  int32_t n_units, batch, row0;
+  int32_t n_units, batch, row0, n_q_heads;
   int64_t t0, n;
   const uint8_t* arena;           // E4M3 codes, one row of D bytes per arena row
   const float* arena_scales;      // per arena row
-  __nv_bfloat16* ring_codes;      // staging rows x D (V rows: fp16 bits)
-  float* ring_scales;             // per staging row (K rows)
+  uint16_t* ring;                 // staging rows x D, fp16
+  const __nv_bfloat16* q;         // chunk input [batch][n][n_q_heads][D]
   const __nv_bfloat16* k;         // chunk input [batch][n][n_units][D]
   const __nv_bfloat16* v;
-  __nv_bfloat16* k_codes;         // chunk K code values, same layout
-  __nv_bfloat16* v_codes;         // chunk V rows dequantized (fp16 bits)
-  float* k_scales;                // [n_units][batch * n + 128]
-  int64_t chunk_scale_stride;
+  uint16_t* q16;                  // the same layouts, fp16
+  uint16_t* k16;
+  uint16_t* v16;
   Fp8StageUnit u[kMaxKvHeads];
 };
 
@@ -175,7 +168,7 @@ cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& k_map,
                           bool fp8 = false);
 cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cudaStream_t s);
 cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s);
-// fp8: K/V tiles are staged 8-bit rows (bf16 code values) with row scales in p
+// fp8: q and the K/V tiles are staged 8-bit-cache rows in fp16 (fp16 mmas)
 cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtensorMap& q_map,
                               const CUtensorMap& ck_map, const CUtensorMap& cv_map,
                               const CUtensorMap& ring_map, cudaStream_t s, bool fp8 = false);

@@ -36,7 +36,10 @@ namespace hwkv {
 
 namespace {
 
-template <int D, int BN, int KST, int VST, int QT, int SBUF, int CTAS, bool PS, bool SC>
+// D head_dim; BN keys per tile; KST / VST K and V tile buffers; QT query tiles per
+// CTA; SBUF S buffers per query tile; CTAS resident CTAs per SM; PS P written over
+// its S columns; F16 q, K and V (and P) in fp16 instead of bf16 (staged 8-bit cache).
+template <int D, int BN, int KST, int VST, int QT, int SBUF, int CTAS, bool PS, bool F16>
 struct TcCfg {
   static constexpr int kSoftmaxWarps = 4 * QT;      // one warpgroup per query tile
   // warp 0 TMA producer, warp 1 QK^T issuer, warps 2 .. 2 + 4 QT - 1 softmax, last warp PV issuer
@@ -61,12 +64,8 @@ struct TcCfg {
   static constexpr int kNumBars = 2 * KST + 2 * VST + 2 * QT * SBUF + 2 * kPBars + 4;
   static constexpr int kBarBytes = 512;
   static_assert(8 * kNumBars + 4 <= kBarBytes, "barriers and the TMEM address slot");
-  // SC (8-bit cache format): K tiles of E4M3 code values with fp32 row scales (per
-  // query tile, two key tiles' scales in shared memory), V tiles of dequantized
-  // rows in fp16 and P in fp16
-  static constexpr int kScaleBytes = SC ? QT * 2 * BN * 4 : 0;
   // the dynamic shared memory window starts 1024-aligned (the kernel checks it)
-  static constexpr int kSmem = kQBytes + (KST + VST) * kTileBytes + kBarBytes + kScaleBytes;
+  static constexpr int kSmem = kQBytes + (KST + VST) * kTileBytes + kBarBytes;
   static_assert(kSmem * CTAS <= 232448 - 1024 * (CTAS - 1), "shared memory per SM");
   static constexpr int kTmemNeed = PS ? kColO + QT * D : kColO + QT * D + QT * BN / 2;
   // first P column of query tile t for key tile j
@@ -195,13 +194,13 @@ __device__ __forceinline__ bool warp_wait_or_abort(uint64_t* bar, uint32_t parit
 
 }  // namespace
 
-template <int D, int BN, int KST, int VST, int QT, int SBUF, int CTAS, bool PS, bool SC>
-__global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>::kThreads, CTAS)
+template <int D, int BN, int KST, int VST, int QT, int SBUF, int CTAS, bool PS, bool F16>
+__global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16>::kThreads, CTAS)
     prefill_tc_kernel(const __grid_constant__ CUtensorMap q_map,
                       const __grid_constant__ CUtensorMap ck_map,
                       const __grid_constant__ CUtensorMap cv_map,
                       const __grid_constant__ CUtensorMap ring_map, const PrefillParams p) {
-  using C = TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>;
+  using C = TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // the 128-byte swizzle atoms need a 1024-aligned base; stop before any copy if
   // the launch ever provides less
@@ -229,8 +228,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
   uint64_t* o_full = q_full + 1;
   uint64_t* drain = o_full + 1;               // [2] each issuer's mmas done
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
-  // [QT][2 key tiles][BN] K row scales (SC only)
-  float* scale_smem = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + C::kBarBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = p.group;
@@ -361,7 +358,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
     // a barrier stops feeding the tensor core, and a 128 x 64 x 16 or 128 x 128 x 16
     // mma is too short to cover that wait from one thread's queue alone.
     if (lane == 0) {
-      constexpr uint32_t idesc_qk = idesc_bf16_f32(128, BN, false);
+      constexpr uint32_t idesc_qk = F16 ? idesc_f16_f32(128, BN, false) : idesc_bf16_f32(128, BN, false);
       const uint32_t q_base = smem_u32(sQ);
       wait_or_abort(q_full, 0, p.err, aborted);
       uint32_t j = 0;
@@ -404,7 +401,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
   } else if (warp == 2 + C::kSoftmaxWarps) {
     // ------------------------------------------------------------- PV issuer
     if (lane == 0) {
-      constexpr uint32_t idesc_pv = SC ? idesc_f16_f32(128, D, true) : idesc_bf16_f32(128, D, true);
+      constexpr uint32_t idesc_pv = F16 ? idesc_f16_f32(128, D, true) : idesc_bf16_f32(128, D, true);
       uint32_t j = 0;
       int hist;
       int32_t j0;
@@ -446,7 +443,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
     const int32_t W = seq.W;
     const int32_t lo_r = W == 0 ? 0 : (pr - W + 1 > 0 ? pr - W + 1 : 0);  // first visible key
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
-    const int64_t krow_base = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;  // ring rows (SC scales)
     const float c = p.scale_log2;
     float m_used = -INFINITY, l = 0.f;  // running max (log2 units) and sum of weights
     uint32_t j = 0;
@@ -483,23 +479,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
       }
       const bool full_vis = (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);
       const bool warp_full = __all_sync(0xffffffffu, full_vis);  // warp-uniform fast path
-      // SC: the tile's K row scales, 32 per warp of the warpgroup, read before the
-      // S wait and put in shared memory after it (two tiles' worth per warpgroup: a
-      // barrier per tile keeps a buffer from being rewritten while it is read)
-      float ks_e = 0.f;
-      const int sc_e = ((warp - 2) & 3) * 32 + lane;
-      if constexpr (SC) {
-        if (sc_e < BN)
-          ks_e = hist ? __ldg(p.k_scale_ring + krow_base + j0 + sc_e)
-                      : __ldg(p.k_scale_chunk + (int64_t)h * p.chunk_scale_stride +
-                              (int64_t)b * n_chunk + j0 + sc_e);
-      }
       if (warp_wait_or_abort(&s_full[tq * SBUF + sb], (j / SBUF) & 1u, p.err, aborted)) tc_fence_after();
-      float* ks_s = scale_smem + (tq * 2 + (int)(j & 1)) * BN;
-      if constexpr (SC) {
-        if (sc_e < BN) ks_s[sc_e] = ks_e;
-        asm volatile("bar.sync %0, 128;" ::"r"(1 + tq) : "memory");
-      }
       // The S row in chunks of 64 columns: pass 1 takes the row max, pass 2 the
       // weights, the row sum and P. With one chunk the registers carry over; with
       // more the chunk is read from TMEM again (P over S overwrites only columns
@@ -510,16 +490,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
         tmem_ld32(t_lane + colS + sb * BN + ch * 64, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
         tmem_ld32(t_lane + colS + sb * BN + ch * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
         tmem_ld_wait();
-        if constexpr (SC) {  // logits of code values times the key row's scale
-#pragma unroll
-          for (int e = 0; e < 64; e += 4) {
-            const float4 k4 = *reinterpret_cast<const float4*>(ks_s + ch * 64 + e);
-            sv[e] = __float_as_uint(__uint_as_float(sv[e]) * k4.x);
-            sv[e + 1] = __float_as_uint(__uint_as_float(sv[e + 1]) * k4.y);
-            sv[e + 2] = __float_as_uint(__uint_as_float(sv[e + 2]) * k4.z);
-            sv[e + 3] = __float_as_uint(__uint_as_float(sv[e + 3]) * k4.w);
-          }
-        }
         if (!warp_full) {  // masked logits -> -inf (weight 0)
 #pragma unroll
           for (int e = 0; e < 64; ++e) {
@@ -594,8 +564,8 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
           const float2 y = fma2(make_float2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), c2, nb2);
           const float2 w = make_float2(ex2(y.x), ex2(y.y));
           if (e & 2) s2b = add2(s2b, w); else s2a = add2(s2a, w);
-          // in place: index e / 2 was already read; fp16 against fp16 V rows (SC)
-          sv[e / 2] = SC ? pack_f16(w.x, w.y) : pack_bf16(w.x, w.y);
+          // in place: index e / 2 was already read; P in the operands' type
+          sv[e / 2] = F16 ? pack_f16(w.x, w.y) : pack_bf16(w.x, w.y);
         }
         if constexpr (!PS) {
           // P is single-buffered apart from S: the previous PV must have read it
@@ -639,17 +609,17 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>
   if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
 }
 
-template <int D, int BN, int KST, int VST, int QT, int SBUF, int CTAS, bool PS, bool SC>
+template <int D, int BN, int KST, int VST, int QT, int SBUF, int CTAS, bool PS, bool F16>
 static cudaError_t launch_tc(const PrefillParams& p, const CUtensorMap& qm, const CUtensorMap& km,
                              const CUtensorMap& vm, const CUtensorMap& rm, cudaStream_t s) {
-  using C = TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>;
-  cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC>,
+  using C = TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16>;
+  cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
   if (e != cudaSuccess) return e;
   const int QP = 128 / p.group;
   const int64_t n_qblocks = (p.n + QP - 1) / QP;
   dim3 grid((unsigned)((n_qblocks + QT - 1) / QT), (unsigned)p.n_units, (unsigned)p.batch);
-  prefill_tc_kernel<D, BN, KST, VST, QT, SBUF, CTAS, PS, SC><<<grid, C::kThreads, C::kSmem, s>>>(qm, km, vm, rm, p);
+  prefill_tc_kernel<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16><<<grid, C::kThreads, C::kSmem, s>>>(qm, km, vm, rm, p);
   return cudaGetLastError();
 }
 
@@ -659,9 +629,9 @@ cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtens
                               const CUtensorMap& ck_map, const CUtensorMap& cv_map,
                               const CUtensorMap& ring_map, cudaStream_t s, bool fp8) {
   if (p.n == 0) return cudaSuccess;
-  if (fp8) {  // staged 8-bit cache: code values plus row scales (head_dim 128 and 256)
+  if (fp8) {  // staged 8-bit cache: q, K and V tiles in fp16 (head_dim 128 and 256)
     switch (head_dim) {
-      case 128: return launch_tc<128, 128, 2, 2, 2, 1, 1, true, true>(p, q_map, ck_map, cv_map, ring_map, s);
+      case 128: return launch_tc<128, 128, 3, 2, 2, 1, 1, true, true>(p, q_map, ck_map, cv_map, ring_map, s);
       case 256: return launch_tc<256, 64, 3, 2, 1, 2, 1, false, true>(p, q_map, ck_map, cv_map, ring_map, s);
       default: return cudaErrorInvalidValue;
     }

@@ -471,19 +471,20 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
     if (e != cudaSuccess) return fail(HWKV_ECUDA, "prefill launch: %s", cudaGetErrorString(e));
   } else {
     // 8-bit cache: attention reads every key as stored (code x row scale), the
-    // chunk's own rows included. The visible ring rows are staged and the chunk
-    // quantized as the append will store it: K as bf16 code values (exact) whose
-    // scales the kernel applies to the logits in fp32, V dequantized in fp16.
-    if (!c->pol.head_dim || (d != 128 && d != 256))
-      return fail(HWKV_EUNSUPPORTED, "8-bit prefill needs head_dim 128 or 256");
+    // chunk's own rows included. The held ring rows are staged dequantized and the
+    // chunk quantized as the append will store it, then dequantized; with q they
+    // go through the tensor cores in fp16 (11 significant bits).
+    if (d != 128 && d != 256) return fail(HWKV_EUNSUPPORTED, "8-bit prefill needs head_dim 128 or 256");
     Fp8StageParams sp{};
     sp.n_units = H;
     sp.batch = n_rows;
     sp.row0 = row0;
+    sp.n_q_heads = c->pol.n_q_heads;
     sp.t0 = t_rows;
     sp.n = n;
     sp.arena = reinterpret_cast<const uint8_t*>(c->k_base());
     sp.arena_scales = c->scales();
+    sp.q = static_cast<const __nv_bfloat16*>(q);
     sp.k = static_cast<const __nv_bfloat16*>(k);
     sp.v = static_cast<const __nv_bfloat16*>(v);
     int64_t rows = 0;
@@ -492,37 +493,40 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
       sp.u[h] = Fp8StageUnit{u.k_row0, u.v_row0, u.cap, u.stride, u.sink, rows, rows + (int64_t)n_rows * u.cap};
       rows += 2 * (int64_t)n_rows * u.cap;
     }
-    const int64_t cstride = (int64_t)n_rows * n + 128;
-    const size_t ring_code_bytes = align_up((size_t)rows * d * 2, 1024);
-    const size_t ring_scale_bytes = align_up((size_t)(rows + 128) * 4, 1024);
-    const size_t chunk_code_bytes = align_up((size_t)n_rows * n * H * d * 2, 1024);
-    const size_t chunk_scale_bytes = align_up((size_t)H * cstride * 4, 1024);
-    const size_t total = ring_code_bytes + ring_scale_bytes + 2 * chunk_code_bytes + chunk_scale_bytes;
+    const size_t ring_bytes = align_up((size_t)rows * d * 2, 1024);
+    const size_t kv_bytes = align_up((size_t)n_rows * n * H * d * 2, 1024);
+    const size_t q_bytes = align_up((size_t)n_rows * n * c->pol.n_q_heads * d * 2, 1024);
+    const size_t total = ring_bytes + 2 * kv_bytes + q_bytes;
     uint8_t* buf = nullptr;
     e = cudaMallocAsync(reinterpret_cast<void**>(&buf), total, s);
     if (e != cudaSuccess) return fail(HWKV_ENOMEM, "8-bit prefill staging (%zu bytes): %s", total, cudaGetErrorString(e));
-    // zeros where nothing is staged: tiles read past the held rows (masked there,
-    // but a weight of 0 times a non-finite value would still poison the sum)
-    e = cudaMemsetAsync(buf, 0, total, s);
-    sp.ring_codes = reinterpret_cast<__nv_bfloat16*>(buf);
-    sp.ring_scales = reinterpret_cast<float*>(buf + ring_code_bytes);
-    sp.k_codes = reinterpret_cast<__nv_bfloat16*>(buf + ring_code_bytes + ring_scale_bytes);
-    sp.v_codes = reinterpret_cast<__nv_bfloat16*>(buf + ring_code_bytes + ring_scale_bytes + chunk_code_bytes);
-    sp.k_scales = reinterpret_cast<float*>(buf + ring_code_bytes + ring_scale_bytes + 2 * chunk_code_bytes);
-    sp.chunk_scale_stride = cstride;
-    if (e == cudaSuccess) e = launch_fp8_stage(sp, d, s);
-    CUtensorMap ring_map;
+    sp.ring = reinterpret_cast<uint16_t*>(buf);
+    sp.k16 = reinterpret_cast<uint16_t*>(buf + ring_bytes);
+    sp.v16 = reinterpret_cast<uint16_t*>(buf + ring_bytes + kv_bytes);
+    sp.q16 = reinterpret_cast<uint16_t*>(buf + ring_bytes + 2 * kv_bytes);
+    e = launch_fp8_stage(sp, d, s);
+    CUtensorMap ring_map, q16_map;
     CUresult r = CUDA_SUCCESS;
     if (e == cudaSuccess) {
       const cuuint64_t gdim[2] = {(cuuint64_t)d, (cuuint64_t)rows};
       const cuuint64_t gstride[1] = {(cuuint64_t)d * 2};
       const cuuint32_t box[2] = {64u, (cuuint32_t)kStageTokens};
       const cuuint32_t es2[2] = {1, 1};
-      r = encode(&ring_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, sp.ring_codes, gdim, gstride, box, es2,
+      r = encode(&ring_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, sp.ring, gdim, gstride, box, es2,
                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-      if (r == CUDA_SUCCESS) r = encode_chunk(&ck_map, sp.k_codes);
-      if (r == CUDA_SUCCESS) r = encode_chunk(&cv_map, sp.v_codes);
+      // the staged copies have the input layouts; the maps only move 2-byte elements
+      if (r == CUDA_SUCCESS) r = encode_chunk(&ck_map, sp.k16);
+      if (r == CUDA_SUCCESS) r = encode_chunk(&cv_map, sp.v16);
+      if (r == CUDA_SUCCESS) {
+        const cuuint64_t dim[3] = {(cuuint64_t)d, (cuuint64_t)c->pol.n_q_heads,
+                                   (cuuint64_t)n_rows * (cuuint64_t)n};
+        const cuuint64_t str[2] = {(cuuint64_t)d * 2, (cuuint64_t)c->pol.n_q_heads * d * 2};
+        const cuuint32_t qbox[3] = {64, (cuuint32_t)G, (cuuint32_t)QP};
+        r = encode(&q16_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, sp.q16, dim, str, qbox, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      }
     }
     if (e == cudaSuccess && r == CUDA_SUCCESS) {
       for (int h = 0; h < H; ++h) {
@@ -531,10 +535,7 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
         p.u[h].stride = sp.u[h].cap;
       }
       p.row0 = 0;
-      p.k_scale_ring = sp.ring_scales;
-      p.k_scale_chunk = sp.k_scales;
-      p.chunk_scale_stride = cstride;
-      e = launch_prefill_tc(p, d, q_map, ck_map, cv_map, ring_map, s, true);
+      e = launch_prefill_tc(p, d, q16_map, ck_map, cv_map, ring_map, s, true);
     }
     const cudaError_t ef = cudaFreeAsync(buf, s);
     if (r != CUDA_SUCCESS) return fail(HWKV_ECUDA, "8-bit prefill tensor maps rejected (%d)", (int)r);
