@@ -309,15 +309,35 @@ def run_gpu(args, wl, world, rank, local, fp8=False):
         host_inputs.append((q.cpu().pin_memory(), k.cpu().pin_memory(), v.cpu().pin_memory()))
     stream.synchronize()
 
+    # Copies overlap the decode: a copy stream brings layer l's q/k/v in while
+    # earlier layers decode, another takes layer l's output out while later ones
+    # run; the step ends when the last output has reached the host. The next
+    # step's copies start only after this step's end (they reuse the buffers).
+    copy_in, copy_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in range(L)]
+    ev_out = [torch.cuda.Event() for _ in range(L)]
+    ev_start, ev_done = torch.cuda.Event(), torch.cuda.Event()
+
     def e2e_step(i):
         qh, kh, vh = host_inputs[i]
-        q_d.copy_(qh, non_blocking=True)
-        k_d.copy_(kh, non_blocking=True)
-        v_d.copy_(vh, non_blocking=True)
+        ev_start.record(stream)
+        copy_in.wait_event(ev_start)
+        with torch.cuda.stream(copy_in):
+            for layer in range(L):
+                q_d[layer].copy_(qh[layer], non_blocking=True)
+                k_d[layer].copy_(kh[layer], non_blocking=True)
+                v_d[layer].copy_(vh[layer], non_blocking=True)
+                ev_in[layer].record(copy_in)
         for layer in range(L):
+            stream.wait_event(ev_in[layer])
             hwkv.hwkv_decode_step(cache, layer, q_d[layer], k_d[layer], v_d[layer], scale,
                                   out[layer], s)
-        o_h.copy_(out, non_blocking=True)
+            ev_out[layer].record(stream)
+            copy_out.wait_event(ev_out[layer])
+            with torch.cuda.stream(copy_out):
+                o_h[layer].copy_(out[layer], non_blocking=True)
+        ev_done.record(copy_out)
+        stream.wait_event(ev_done)
 
     for i in range(2):
         e2e_step(i)
