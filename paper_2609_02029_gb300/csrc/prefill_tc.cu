@@ -20,14 +20,19 @@
 //   warp 1      QK^T issuer (one thread): per key tile, S_t = Q_t K^T for each
 //               query tile t into its TMEM tile (128 x BN fp32, SBUF-buffered)
 //   warps 2+    softmax, one warpgroup per query tile: thread r owns TMEM lane
-//               r = query row r, so the row max and sum are thread-local; P goes
-//               back to TMEM as bf16 and is the tensor-memory A operand of the
-//               PV mma; O is rescaled in TMEM only when a row's running max
-//               grows by more than 2^8 (the final O / l uses the same
-//               reference, so the result is exact).
+//               r = query row r, so the row max and sum are thread-local; the S
+//               row is read in 64-column chunks (row max, then weights, sum and
+//               P); P goes back to TMEM as bf16 pairs (with PS over the first half
+//               of its own S columns) and is the tensor-memory A operand of the PV
+//               mma; O is rescaled in TMEM only when a row's running max grows by
+//               more than 2^8 (the final O / l uses the same reference, so the
+//               result is exact)
 //   last warp   PV issuer (one thread): O_t += P_t V per key tile (128 x D fp32)
-// While the softmax warps work on key tile j the tensor core computes S of the
-// next key tile and the PV products of the tile before.
+// Two issuing threads keep the tensor core fed while one of them waits on a
+// barrier (a wait after an mma batch drains that thread's short mma queue). With
+// P over one S buffer a tile's next QK^T waits for its PV, so the QT tiles of a CTA
+// overlap each other's softmax and products; without PS (SBUF buffers, P apart) a
+// tile's next QK^T only waits until its softmax has read S.
 // All waits are bounded; a thread that gives up stops waiting and issuing but
 // keeps walking the tile sequence, so every role reaches the TMEM release.
 #include "hwkv_internal.cuh"
