@@ -73,6 +73,13 @@ struct TcCfg {
   static constexpr int kSmem = kQBytes + (KST + VST) * kTileBytes + kBarBytes;
   static_assert(kSmem * CTAS <= 232448 - 1024 * (CTAS - 1), "shared memory per SM");
   static constexpr int kTmemNeed = PS ? kColO + QT * D : kColO + QT * D + QT * BN / 2;
+  // P of key chunk ch (64 keys = 32 columns) relative to col_p: chunk 0 first; with
+  // PS and two chunks the last chunk's P goes over the second half of its own S
+  // columns (already in registers when its P is written), every other chunk's P
+  // over the first half of chunk 0's S columns
+  __device__ static constexpr uint32_t p_chunk_col(int ch) {
+    return (PS && BN == 128 && ch == 1) ? 96u : (uint32_t)(ch * 32);
+  }
   // first P column of query tile t for key tile j
   __device__ static constexpr uint32_t col_p(int t, uint32_t j) {
     return PS ? (uint32_t)(kColS + (t * SBUF + (int)(j % SBUF)) * BN)
@@ -178,6 +185,13 @@ struct KeySeq {
     return false;
   }
 };
+
+// max of three floats in one instruction
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
 
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, int* err,
                                               bool& aborted) {
@@ -421,7 +435,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
 #pragma unroll
             for (int kk = 0; kk < BN / 16; ++kk) {  // 16 keys = 8 packed P columns
               const uint64_t bd = smem_desc_sw128(v_base + kk * 2048, C::kKVSlab, 1024);
-              umma_bf16_tmem_a(tmem + C::kColO + t * D, tmem + C::col_p(t, j) + kk * 8, bd,
+              umma_bf16_tmem_a(tmem + C::kColO + t * D, tmem + C::col_p(t, j) + C::p_chunk_col(kk / 4) + (kk % 4) * 8, bd,
                                idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
             }
             umma_commit(&pv_done[C::p_bar(t, j)]);
@@ -512,7 +526,10 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
         for (int ch = 0; ch < kChunks; ++ch) {
           load_chunk(ch);
 #pragma unroll
-          for (int e = 0; e < 64; ++e) m4[e & 3] = fmaxf(m4[e & 3], __uint_as_float(sv[e]));
+          for (int e = 0; e < 64; e += 8)
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              m4[i] = fmax3(m4[i], __uint_as_float(sv[e + i]), __uint_as_float(sv[e + 4 + i]));
         }
         mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
         mx *= c;
@@ -560,9 +577,11 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
       // weights 2^(z c - m) (masked logits are -inf: weight 0); the exponent
       // arguments and the row sum in packed fp32 pairs; P as bf16 pairs
       float2 s2a = make_float2(0.f, 0.f), s2b = make_float2(0.f, 0.f);
+      // the last chunk is still in registers: it goes first; the others are read again
 #pragma unroll
-      for (int ch = 0; ch < kChunks; ++ch) {
-        if (kChunks > 1) load_chunk(ch);
+      for (int cc = 0; cc < kChunks; ++cc) {
+        const int ch = (cc + kChunks - 1) % kChunks;
+        if (cc > 0) load_chunk(ch);
         const float2 c2 = make_float2(c, c), nb2 = make_float2(-bias, -bias);
 #pragma unroll
         for (int e = 0; e < 64; e += 2) {
@@ -578,7 +597,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
             tc_fence_after();
           rescale_o();
         }
-        tmem_st32(t_lane + C::col_p(tq, j) + ch * 32, *reinterpret_cast<const uint32_t(*)[32]>(&sv[0]));
+        tmem_st32(t_lane + C::col_p(tq, j) + C::p_chunk_col(ch), *reinterpret_cast<const uint32_t(*)[32]>(&sv[0]));
       }
       tmem_st_wait();
       float s4[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
