@@ -447,7 +447,7 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
         const int64_t row_in = ti.s_new - (ti.start + (int64_t)st * kStageTokens);
         if constexpr (FP8) {
          if (row_in >= w * 16 && row_in < w * 16 + 16) {
-          // quantise as the append does: amax over the row, s = amax / 448, codes of x / s
+          // quantise as the append does (the same row helper)
           constexpr int PER = D / 32;
           const int r = (int)row_in;
 #pragma unroll
@@ -462,26 +462,12 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
               const uint2 v = *reinterpret_cast<const uint2*>(src);
               raw[0] = v.x; raw[1] = v.y;
             }
-            float x[PER], amax = 0.f;
+            float x[PER];
 #pragma unroll
-            for (int j = 0; j < PER; ++j) {
+            for (int j = 0; j < PER; ++j)
               x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
-              amax = fmaxf(amax, fabsf(x[j]));
-            }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1)
-              amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-            const float sc = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
             uint32_t cw[PER / 4];
-#pragma unroll
-            for (int j = 0; j < PER; j += 4) {
-              uint32_t c01 = 0, c23 = 0;
-              if (amax > 0.f) {
-                c01 = f32x2_to_e4m3x2(__fdiv_rn(x[j], sc), __fdiv_rn(x[j + 1], sc));
-                c23 = f32x2_to_e4m3x2(__fdiv_rn(x[j + 2], sc), __fdiv_rn(x[j + 3], sc));
-              }
-              cw[j / 4] = c01 | (c23 << 16);
-            }
+            const float sc = e4m3_quantize_row_warp<PER>(x, cw);
             const int64_t ring = (kv ? ti.v_row : ti.k_row) - ti.start + ti.s_new;
             uint8_t* g = reinterpret_cast<uint8_t*>(p.arena) + ring * D + lane * PER;
             const int c0 = lane * PER;  // first channel of this lane
