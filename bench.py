@@ -719,6 +719,7 @@ def main():
               "dtype": "fp8-e4m3 KV" if args.kv == "fp8" else "bf16", "data": "synthetic",
               "config": {"workload": "prefill64k", "kv_format": args.kv}, "ms": pre["ms"],
               "flops": pre["flops"], "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst,
+              "frac_of_sustained": pre["tflops"] / tf_sust,
               "peak_source": peak_src})
         return
     r = run_gpu(args, wl, world, rank, local, fp8=args.kv == "fp8")
@@ -783,6 +784,8 @@ def main():
     if pre is not None:
         line["prefill"] = {"workload": "prefill64k", "tflops": pre["tflops"],
                            "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst,
+                           "peak_tflops_sustained": tf_sust,
+                           "frac_of_sustained": pre["tflops"] / tf_sust,
                            "peak_source": peak_src, "ms": pre["ms"],
                            "tokens_per_s": pre["tokens_per_s"], "flops": pre["flops"]}
         if pre8 is not None:
