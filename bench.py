@@ -463,7 +463,8 @@ def run_prefill(args, local, fp8=False):
     arena = torch.empty(nbytes, dtype=torch.uint8, device=dev)
     reps = []
     flops = sum(prefill_flops(wl, c * n, n) for c in range(chunks))
-    for rep in range(1 + args.prefill_reps):
+    warm = 3 if args.prefill_reps > 1 else 1  # a single rep is the profiling case
+    for rep in range(warm + args.prefill_reps):
         cache = hwkv.hwkv_alloc(pol, arena, nbytes, s)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
@@ -473,7 +474,7 @@ def run_prefill(args, local, fp8=False):
         e1.synchronize()
         hwkv.hwkv_sync_check(cache)
         hwkv.hwkv_free(cache)
-        if rep > 0:
+        if rep >= warm:
             reps.append(e0.elapsed_time(e1))
     ms = float(np.median(reps))
     del q, k, v, out, arena
@@ -651,7 +652,7 @@ def main():
                     help="cache format of the timed decode (fp8: E4M3 codes + row scales)")
     ap.add_argument("--no-fp8", action="store_true",
                     help="skip the secondary 8-bit-cache decode measurement")
-    ap.add_argument("--prefill-reps", type=int, default=3)
+    ap.add_argument("--prefill-reps", type=int, default=5)
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-calib", action="store_true")
