@@ -614,23 +614,31 @@ class OracleSample:
         """Whole-step time, scaling the sample by keys attended (cost is linear in keys)."""
         return sec * self.keys_all / max(keys, 1)
 
-    def describe(self, n, keys, sec):
+    def describe(self, n, keys, sec, passes=1):
+        rep = " (mean of %d passes)" % passes if passes > 1 else ""
         return ("%d of %d (layer, batch row, KV head) units of one decode step at t=%d, "
-                "%d of %d keys, fp64 oracle %.2f s on %d threads, scaled by keys to the full "
-                "step" % (n, len(self.units_all), self.t, keys, self.keys_all, sec, self.cores))
+                "%d of %d keys, fp64 oracle %.2f s%s on %d threads, scaled by keys to the full "
+                "step" % (n, len(self.units_all), self.t, keys, self.keys_all, sec, rep,
+                          self.cores))
 
 
-def cpu_baseline(wl, max_ctx, t, budget_s=15.0):
-    """Oracle tokens/s on this host's cores from a bounded sample of one step."""
+def cpu_baseline(wl, max_ctx, t, budget_s=15.0, min_s=10.0):
+    """Oracle tokens/s on this host's cores from a bounded sample of one step: the
+    sampled units are run again until about `min_s` seconds of oracle work are timed."""
     cores = os.cpu_count() or 1
     samp = OracleSample(wl, max_ctx, t, max_units=8 * cores)
     sec, n, keys = samp.run()
     if sec > budget_s and n > cores:  # keep the timed work bounded
         m = max(cores, int(n * budget_s / sec))
         sec, n, keys = samp.run(m)
+    total, passes = sec, 1
+    while total < min_s and passes < 64:
+        total += samp.run(n)[0]
+        passes += 1
+    sec = total / passes
     step_s = samp.step_seconds(sec, keys)
     return {"value": wl.batch / step_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": samp.describe(n, keys, sec)}
+            "sample": samp.describe(n, keys, sec, passes)}
 
 
 # ------------------------------------------------------------------ main
