@@ -496,7 +496,10 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
           }
         }
       }
-      const bool full_vis = (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);
+      // A row that carries no (position, head) (the tile's last 128 mod G rows, or
+      // rows past the chunk) counts as fully visible: its output is never stored and
+      // it never rescales O, so it does not hold its warp on the masked path.
+      const bool full_vis = !row_ok || (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);
       const bool warp_full = __all_sync(0xffffffffu, full_vis);  // warp-uniform fast path
       if (warp_wait_or_abort(&s_full[tq * SBUF + sb], (j / SBUF) & 1u, p.err, aborted)) tc_fence_after();
       // The S row in chunks of 64 columns: pass 1 takes the row max, pass 2 the
@@ -541,7 +544,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
         if (lane == 0) mbar_arrive(&s_free[tq * SBUF + sb]);
       }
       const float m_new = fmaxf(m_used, mx);
-      const bool resc = m_new - m_used > 8.f;  // false while both are -inf
+      const bool resc = row_ok && m_new - m_used > 8.f;  // false while both are -inf
       float alpha = 1.f;
       if (resc) {
         alpha = ex2(m_used - m_new);
