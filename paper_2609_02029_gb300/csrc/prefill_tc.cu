@@ -47,8 +47,14 @@ namespace {
 template <int D, int BN, int KST, int VST, int QT, int SBUF, int CTAS, bool PS, bool F16>
 struct TcCfg {
   static constexpr int kSoftmaxWarps = 4 * QT;      // one warpgroup per query tile
-  // warp 0 TMA producer, warp 1 QK^T issuer, warps 2 .. 2 + 4 QT - 1 softmax, last warp PV issuer
-  static constexpr int kThreads = 96 + 32 * kSoftmaxWarps;
+  // One thread's TMA tile copies reach ~45 B/clk into an SM, two threads' ~72. With
+  // one query tile per CTA a key tile's K and V (4 d B per key) feed half the rows
+  // they feed with two, so V tiles get a producer warp of their own.
+  static constexpr bool kSplitV = QT == 1;
+  // warp 0 TMA producer (K only with kSplitV), warp 1 QK^T issuer, warps 2 .. 2 + 4 QT - 1
+  // softmax, warp 2 + 4 QT PV issuer, then (kSplitV) the V producer
+  static constexpr int kVWarp = 3 + kSoftmaxWarps;
+  static constexpr int kThreads = 96 + 32 * kSoftmaxWarps + (kSplitV ? 32 : 0);
   static_assert(BN % 32 == 0 && D % 32 == 0, "TMEM loads of 32 columns");
   static constexpr int kSlabs = D / 64;
   static constexpr int kQSlab = 128 * 128;             // 128 rows x 128 B
@@ -301,7 +307,64 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
   seq.init(u, t0, n_chunk, p0, p_last);
   bool aborted = false;
 
-  if (warp == 0) {
+  if (C::kSplitV && (warp == 0 || warp == C::kVWarp)) {
+    // ------------------------------------------------- K and V producers (kSplitV)
+    // warp 0 copies Q and the K tiles, warp kVWarp the V tiles, each walking the key
+    // sequence into its own ring
+    if (lane == 0) {
+      const bool is_k = warp == 0;
+      if (is_k) {
+        prefetch_tensormap(&q_map);
+        prefetch_tensormap(&ck_map);
+      }
+      prefetch_tensormap(&cv_map);
+      prefetch_tensormap(&ring_map);
+      if (is_k) {
+        // the query tile's box is copied whole, so the byte count is fixed
+        mbar_arrive_expect_tx(q_full, (uint32_t)(QT * C::kSlabs * rows_valid * 128));
+#pragma unroll
+        for (int t = 0; t < QT; ++t) {
+          const int32_t qrow = (int32_t)((int64_t)b * p.n + (int64_t)(qb0 + t) * QP);
+#pragma unroll
+          for (int sl = 0; sl < C::kSlabs; ++sl)
+            tma_load_3d(sQ + t * C::kQTile + sl * C::kQSlab, &q_map, sl * 64, h * G, qrow, q_full);
+        }
+      }
+      const int nbuf = is_k ? KST : VST;
+      uint64_t* full = is_k ? k_full : v_full;
+      uint64_t* empty = is_k ? k_empty : v_empty;
+      uint8_t* buf = is_k ? sK : sV;
+      const CUtensorMap* cmap = is_k ? &ck_map : &cv_map;
+      const int64_t row0 = (is_k ? u.k_row0 : u.v_row0) + (int64_t)(p.row0 + b) * u.stride;
+      uint32_t it = 0;
+      int hist;
+      int32_t j0;
+      while (seq.next(hist, j0)) {
+        const int s = it % nbuf;
+        if (wait_or_abort(&empty[s], ((it / nbuf) & 1u) ^ 1u, p.err, aborted)) {
+          uint8_t* d = buf + s * C::kTileBytes;
+          mbar_arrive_expect_tx(&full[s], C::kTileBytes);
+#pragma unroll
+          for (int sl = 0; sl < C::kSlabs; ++sl) {
+#pragma unroll
+            for (int hf = 0; hf < BN / 64; ++hf) {
+              const uint32_t off = sl * C::kKVSlab + hf * 64 * 128;
+              if (hist)
+                tma_load_2d(d + off, &ring_map, sl * 64, (int32_t)(row0 + j0 + hf * 64), &full[s]);
+              else
+                tma_load_3d(d + off, cmap, sl * 64, h, (int32_t)((int64_t)b * p.n + j0 + hf * 64),
+                            &full[s]);
+            }
+          }
+        }
+        ++it;
+      }
+      // every copy this thread issued has landed before shared memory can go away
+      bool late = false;
+      for (uint32_t j = it > (uint32_t)nbuf ? it - nbuf : 0u; j < it; ++j)
+        wait_or_abort(&full[j % nbuf], (j / nbuf) & 1u, p.err, late);
+    }
+  } else if (warp == 0) {
     // ---------------------------------------------------------------- producer
     if (lane == 0) {
       prefetch_tensormap(&q_map);
