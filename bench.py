@@ -432,16 +432,17 @@ def sum_range(a, b):
     return 0 if b < a else (a + b) * (b - a + 1) // 2
 
 
-def run_prefill(args, local, fp8=False):
-    """prefill64k: the 64K prompt as eight 8,192-token chunks through hwkv_prefill.
-    With fp8 the cache holds E4M3 codes + row scales; the timed region then also
-    covers the per-call staging of the visible rows and the 8-bit append."""
+def run_prefill(args, local, fp8=False, workload="prefill64k"):
+    """A whole prompt in 8,192-token chunks through hwkv_prefill: prefill64k (64K
+    tokens, head_dim 128) or single32k (32K tokens, head_dim 256). With fp8 the cache
+    holds E4M3 codes + row scales; the timed region then also covers the per-call
+    staging of the visible rows and the 8-bit append."""
     import torch
 
     import hwkv_gen
     import paper_2609_02029_gb300 as hwkv
 
-    wl = workloads.make("prefill64k")
+    wl = workloads.make(workload)
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     s = stream.cuda_stream
@@ -665,7 +666,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-calib", action="store_true")
     ap.add_argument("--prefill-only", action="store_true",
-                    help="run only the 64K prefill measurement (profiling)")
+                    help="run only a prefill measurement (profiling)")
+    ap.add_argument("--prefill-workload", default="prefill64k", choices=["prefill64k", "single32k"],
+                    help="prompt of --prefill-only")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: keep the first N layers (the reported workload is "
                          "the full one)")
@@ -722,11 +725,11 @@ def main():
         return
 
     if args.prefill_only:
-        pre = run_prefill(args, local, fp8=args.kv == "fp8")
+        pre = run_prefill(args, local, fp8=args.kv == "fp8", workload=args.prefill_workload)
         emit({"metric": "prefill TFLOP/s", "value": pre["tflops"], "unit": "TFLOP/s",
               "n_gpus": 1, "higher_is_better": True,
               "dtype": "fp8-e4m3 KV" if args.kv == "fp8" else "bf16", "data": "synthetic",
-              "config": {"workload": "prefill64k", "kv_format": args.kv}, "ms": pre["ms"],
+              "config": {"workload": args.prefill_workload, "kv_format": args.kv}, "ms": pre["ms"],
               "flops": pre["flops"], "peak_tflops": tf_burst, "frac": pre["tflops"] / tf_burst,
               "frac_of_sustained": pre["tflops"] / tf_sust,
               "peak_source": peak_src})
@@ -737,11 +740,12 @@ def main():
         a8 = argparse.Namespace(**vars(args))
         a8.steps, a8.e2e_steps = min(args.steps, 32), 2
         r8 = run_gpu(a8, wl, world, rank, local, fp8=True)
-    pre = pre8 = None
+    pre = pre8 = pre256 = None
     if not args.no_prefill and rank == 0:
         pre = run_prefill(args, local)
         if not args.no_fp8:
             pre8 = run_prefill(args, local, fp8=True)
+        pre256 = run_prefill(args, local, workload="single32k")
     cal = None
     if rank == 0 and not args.no_calib:
         cal = run_calib(local)
@@ -802,6 +806,13 @@ def main():
                 "tflops": pre8["tflops"], "ms": pre8["ms"], "tokens_per_s": pre8["tokens_per_s"],
                 "note": "same prompt with the cache in E4M3 codes + row scales; each call stages "
                         "q and the held/new K/V rows dequantized in fp16, then appends in 8 bits"}
+        if pre256 is not None:
+            line["prefill"]["head_dim_256"] = {
+                "workload": "single32k", "tflops": pre256["tflops"],
+                "frac": pre256["tflops"] / tf_burst, "ms": pre256["ms"],
+                "tokens_per_s": pre256["tokens_per_s"], "flops": pre256["flops"],
+                "note": "32K prompt in 8K chunks, batch 1, 24q/4kv, head_dim 256, windows "
+                        "{full, 16384, 4096, 1024}"}
     if cal is not None:
         line["seqcalib"] = cal
     if cb is not None:
