@@ -161,6 +161,26 @@ def test_sink_prefill_decode_and_rings():
         r.close()
 
 
+@pytest.mark.parametrize("fmt", [hwkv.HWKV_KV_BF16, hwkv.HWKV_KV_FP8_E4M3])
+def test_sink_prefill_head_dim_256(fmt):
+    # d = 256, 24 query / 4 KV heads (G = 6: 126 rows per 128-row tile): the kernel with one
+    # query tile per CTA and separate K and V copy threads, over sink tiles, wrapped window
+    # regions, a plain window and a full head, with chunks shorter and longer than windows
+    r = RunS(windows=[100, 33, 0, 200], sinks=[4, 31, 0, 0], n_q_heads=24, n_kv_heads=4,
+             head_dim=256, max_ctx=1200, seed=9, kv_format=fmt)
+    try:
+        r.prefill(20)    # inside head 1's sinks
+        r.check_rings()
+        r.prefill(150)   # past every sink region; the window regions wrap
+        r.check_rings()
+        r.prefill(333)   # one chunk longer than every window
+        r.check_rings()
+        r.check_residency()
+        hwkv.hwkv_sync_check(r.cache)
+    finally:
+        r.close()
+
+
 def test_sink_appends_and_graph_step():
     import torch
     # d = 256, 24 query / 4 KV heads: sink heads with several (S, W), a plain window, a full head
