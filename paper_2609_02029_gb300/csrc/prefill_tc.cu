@@ -16,7 +16,9 @@
 // same KV head and streams the union of their key tiles once, so every K/V tile
 // brought into shared memory feeds QT x 128 rows. Warp roles:
 //   warp 0      TMA producer: Q once, then K tiles into a KST-deep ring and
-//               V tiles into a VST-deep ring (K runs ahead of V)
+//               V tiles into a VST-deep ring (K runs ahead of V); with one query
+//               tile per CTA the V tiles come from a producer warp of their own
+//               (after the PV issuer), as one thread's copies cannot feed it
 //   warp 1      QK^T issuer (one thread): per key tile, S_t = Q_t K^T for each
 //               query tile t into its TMEM tile (128 x BN fp32, SBUF-buffered)
 //   warps 2+    softmax, one warpgroup per query tile: thread r owns TMEM lane
