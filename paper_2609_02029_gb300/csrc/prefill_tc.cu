@@ -724,7 +724,7 @@ cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtens
   if (fp8) {  // staged 8-bit cache: q, K and V tiles in fp16 (head_dim 128 and 256)
     switch (head_dim) {
       case 128: return launch_tc<128, 128, 3, 2, 2, 1, 1, true, true>(p, q_map, ck_map, cv_map, ring_map, s);
-      case 256: return launch_tc<256, 64, 3, 2, 1, 2, 1, false, true>(p, q_map, ck_map, cv_map, ring_map, s);
+      case 256: return launch_tc<256, 64, 2, 3, 1, 2, 1, false, true>(p, q_map, ck_map, cv_map, ring_map, s);
       default: return cudaErrorInvalidValue;
     }
   }
@@ -733,7 +733,7 @@ cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtens
     //  P over S>
     case 64: return launch_tc<64, 128, 4, 4, 2, 1, 1, true, false>(p, q_map, ck_map, cv_map, ring_map, s);
     case 128: return launch_tc<128, 128, 3, 2, 2, 1, 1, true, false>(p, q_map, ck_map, cv_map, ring_map, s);
-    case 256: return launch_tc<256, 64, 3, 2, 1, 2, 1, false, false>(p, q_map, ck_map, cv_map, ring_map, s);
+    case 256: return launch_tc<256, 64, 2, 3, 1, 2, 1, false, false>(p, q_map, ck_map, cv_map, ring_map, s);
     default: return cudaErrorInvalidValue;
   }
 }
