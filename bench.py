@@ -485,6 +485,55 @@ def run_prefill(args, local, fp8=False, workload="prefill64k"):
                 tokens_per_s=B * wl.prompt / (ms * 1e-3))
 
 
+# ------------------------------------------------------------ GPU append
+def run_append(local, n=8192, reps=10, warm=3):
+    """hwkv_append of 8,192-token chunks into layer 0 of layers16_112k (batch 16,
+    4 KV heads, d 256, rings of {full, 32768, 8192, 2048, 512} drawn per head):
+    each call reads the chunk's K and V (537 MB, more than L2) and writes the last
+    min(n, cap) tokens of every head into its ring. Algorithmic bytes per call:
+    batch x sum_h min(n, cap_h) x 4d written plus the same read from the input
+    (only the rows that land are read). Full heads hold max_ctx = 14 chunks, so at
+    most 14 calls."""
+    import torch
+
+    import hwkv_gen
+    import paper_2609_02029_gb300 as hwkv
+
+    wl = workloads.make("layers16_112k")
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    s = stream.cuda_stream
+    g = hwkv_gen.desc(wl.seed, wl.per_head_scale)
+    B, Hkv, d = wl.batch, wl.n_kv_heads, wl.head_dim
+    windows = wl.windows[:Hkv]
+    k = torch.empty((B, n, Hkv, d), dtype=torch.bfloat16, device=dev)
+    v = torch.empty_like(k)
+    hwkv_gen.fill_device(g, hwkv_gen.K, 0, B, 0, n, Hkv, d, k.data_ptr(), s)
+    hwkv_gen.fill_device(g, hwkv_gen.V, 0, B, 0, n, Hkv, d, v.data_ptr(), s)
+    pol = hwkv.make_policy(1, Hkv, wl.n_q_heads, d, B, wl.max_ctx, windows)
+    nbytes = hwkv.hwkv_required_bytes(pol)
+    arena = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    cache = hwkv.hwkv_alloc(pol, arena, nbytes, s)
+    caps = [wl.max_ctx if (W == 0 or W >= wl.max_ctx) else W for W in windows]
+    per_call = 2 * B * sum(min(n, c) for c in caps) * 4 * d
+    times = []
+    for i in range(warm + reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        hwkv.hwkv_append(cache, 0, k, v, n, s)
+        e1.record(stream)
+        e1.synchronize()
+        if i >= warm:
+            times.append(e0.elapsed_time(e1))
+    hwkv.hwkv_sync_check(cache)
+    hwkv.hwkv_free(cache)
+    ms = float(np.median(times))
+    del k, v, arena
+    torch.cuda.empty_cache()
+    return {"workload": "layers16_112k layer 0, 8192-token chunks", "ms": ms,
+            "bytes_per_call": per_call, "gbs": per_call / (ms * 1e-3) / 1e9}
+
+
 # ------------------------------------------------------------ GPU SeqCalib
 def run_calib(local, T=131072, P=256, Hkv=4, Hq=24, d=256, windows=(8192, 16384, 32768), reps=3):
     """Candidate replay of one layer's trace: a T-token trace, P query positions
@@ -668,6 +717,8 @@ def main():
     ap.add_argument("--no-calib", action="store_true")
     ap.add_argument("--prefill-only", action="store_true",
                     help="run only a prefill measurement (profiling)")
+    ap.add_argument("--append-only", action="store_true",
+                    help="run only the chunk append measurement (profiling)")
     ap.add_argument("--prefill-workload", default="prefill64k", choices=["prefill64k", "single32k"],
                     help="prompt of --prefill-only")
     ap.add_argument("--layers", type=int, default=0,
@@ -725,6 +776,14 @@ def main():
                       "d2h_bytes_per_step": 0}})
         return
 
+    if args.append_only:
+        a = run_append(local)
+        emit({"metric": "append GB/s", "value": a["gbs"], "unit": "GB/s", "n_gpus": 1,
+              "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+              "config": {"workload": a["workload"]}, "ms": a["ms"],
+              "bytes_per_call": a["bytes_per_call"], "peak": hbm, "frac": a["gbs"] / hbm,
+              "peak_source": peak_src})
+        return
     if args.prefill_only:
         pre = run_prefill(args, local, fp8=args.kv == "fp8", workload=args.prefill_workload)
         emit({"metric": "prefill TFLOP/s", "value": pre["tflops"], "unit": "TFLOP/s",
@@ -747,6 +806,7 @@ def main():
         if not args.no_fp8:
             pre8 = run_prefill(args, local, fp8=True)
         pre256 = run_prefill(args, local, workload="single32k")
+    app = run_append(local) if (not args.no_prefill and rank == 0) else None
     cal = None
     if rank == 0 and not args.no_calib:
         cal = run_calib(local)
@@ -814,6 +874,11 @@ def main():
                 "tokens_per_s": pre256["tokens_per_s"], "flops": pre256["flops"],
                 "note": "32K prompt in 8K chunks, batch 1, 24q/4kv, head_dim 256, windows "
                         "{full, 16384, 4096, 1024}"}
+    if app is not None:
+        line["append"] = {"workload": app["workload"], "gbs": app["gbs"], "frac": app["gbs"] / hbm,
+                          "ms": app["ms"], "bytes_per_call": app["bytes_per_call"],
+                          "note": "hwkv_append alone (the decode step fuses its one-token append); "
+                                  "bytes = rows written + the same rows read"}
     if cal is not None:
         line["seqcalib"] = cal
     if cb is not None:

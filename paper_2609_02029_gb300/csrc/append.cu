@@ -5,9 +5,10 @@
 // Position p of KV head u goes to slot p mod cap_u (with S sink slots: p < S
 // to slot p, later ones to slot S + (p - S) mod (cap_u - S)); every row has its
 // own first position t0 (ragged rows). A new token whose window slot a later
-// token of the same call takes is not written. Block 0 also stores the rows' new lengths in the device length array. One launch covers every KV head and batch row of a layer;
-// each thread moves one 16-byte vector, reads are coalesced over the input
-// [batch][n][heads][d] and writes over the ring rows.
+// token of the same call takes is not written (nor read). Block 0 also stores the
+// rows' new lengths in the device length array. One launch covers every KV head
+// and batch row of a layer (grid y and z); each thread moves 16-byte vectors of the
+// rows that land, reads coalesced within each input row and writes over the ring rows.
 #include "hwkv_internal.cuh"
 
 namespace hwkv {
@@ -15,31 +16,41 @@ namespace hwkv {
 __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
   grid_dep_wait();  // k/v may come from the kernel launched before; the previous
                     // decode of this ring must be done reading before slots are reused
-  if (blockIdx.x == 0 && p.lens != nullptr)  // nothing in this grid reads the lengths
-    for (int b = threadIdx.x; b < p.batch; b += blockDim.x)
+  if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && p.lens != nullptr)
+    for (int b = threadIdx.x; b < p.batch; b += blockDim.x)  // nothing in this grid reads them
       p.lens[p.row0 + b] = (int32_t)(p.t0[b] + p.n);
-  const int64_t vec_per_row = p.d / 8;
-  const int64_t total = (int64_t)p.batch * p.n * p.n_units * vec_per_row;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+  // block (x, h, b): KV head h of batch row b. Of the n new tokens only these land:
+  // the ns that are sink positions (< sink, slot = position) and, of the rest, the
+  // last wr (window-region slots), whose slots follow each other from one base mod wr
+  const int h = blockIdx.y, b = blockIdx.z;
+  const AppendUnit& u = p.u[h];
+  const int64_t n = p.n, t0 = p.t0[b];
+  const int64_t wr = u.cap - u.sink;
+  const int64_t ns = u.sink - t0 <= 0 ? 0 : (u.sink - t0 < n ? u.sink - t0 : n);
+  const int64_t iw = n - wr > ns ? n - wr : ns;  // first new token kept in the window region
+  const int64_t count = ns + (n - iw);
+  const int64_t base = iw < n ? (t0 + iw - u.sink) % wr : 0;  // window slot of token iw
+  const int vpr_log2 = __ffs((int)(p.d / 8)) - 1;  // 16-byte vectors per row: 8, 16 or 32
+  const int64_t vmask = (1 << vpr_log2) - 1;
+  const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;
+  const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.stride;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < (count << vpr_log2);
        e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t vec = e % vec_per_row;
-    int64_t r = e / vec_per_row;
-    const int h = (int)(r % p.n_units);
-    r /= p.n_units;
-    const int64_t i = r % p.n;
-    const int b = (int)(r / p.n);
-    const AppendUnit& u = p.u[h];
-    const int64_t pos = (int64_t)p.t0[b] + i;
-    // a window slot is overwritten within this call if position pos + (cap - sink) comes too
-    if (pos >= u.sink && pos < (int64_t)p.t0[b] + p.n - (u.cap - u.sink)) continue;
-    const int64_t slot = ring_slot(pos, u.cap, u.sink);
-    const int64_t src = ((((int64_t)b * p.n + i) * p.n_units + h) * p.d) + vec * 8;
-    const int64_t krow = u.k_row0 + (int64_t)(p.row0 + b) * u.stride + slot;
-    const int64_t vrow = u.v_row0 + (int64_t)(p.row0 + b) * u.stride + slot;
+    const int64_t j = e >> vpr_log2, vec = e & vmask;
+    int64_t i, slot;
+    if (j < ns) {
+      i = j;
+      slot = t0 + j;
+    } else {
+      i = iw + (j - ns);
+      const int64_t q = base + (j - ns);  // < 2 wr
+      slot = u.sink + (q >= wr ? q - wr : q);
+    }
+    const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * p.d) + vec * 8;
     const uint4 kv = *reinterpret_cast<const uint4*>(p.k + src);
     const uint4 vv = *reinterpret_cast<const uint4*>(p.v + src);
-    *reinterpret_cast<uint4*>(p.k_arena + krow * p.d + vec * 8) = kv;
-    *reinterpret_cast<uint4*>(p.v_arena + vrow * p.d + vec * 8) = vv;
+    *reinterpret_cast<uint4*>(p.k_arena + (krow0 + slot) * p.d + vec * 8) = kv;
+    *reinterpret_cast<uint4*>(p.v_arena + (vrow0 + slot) * p.d + vec * 8) = vv;
   }
 }
 
@@ -237,10 +248,12 @@ cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s) {
   }
   const int64_t total = (int64_t)p.batch * p.n * p.n_units * (p.d / 8);
   if (total == 0) return cudaSuccess;
-  int64_t blocks = (total + 255) / 256;
-  const int64_t cap_blocks = 152 * 16;
-  if (blocks > cap_blocks) blocks = cap_blocks;
-  return launch_pdl(append_kernel, dim3((unsigned)blocks), dim3(256), 0, s, p);
+  // up to 4 vectors per thread for a head that keeps all n tokens; blocks of heads
+  // that keep fewer find no work and return
+  int64_t blocks = (p.n * (p.d / 8) + 1023) / 1024;
+  if (blocks > 65535) blocks = 65535;
+  return launch_pdl(append_kernel, dim3((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch),
+                    dim3(256), 0, s, p);
 }
 
 }  // namespace hwkv
