@@ -13,8 +13,9 @@ metric with each step's q/k/v copied from pinned host memory and the outputs
 read back inside the timed region. `roofline` rates the decode kernel against
 the measured HBM copy bandwidth; `prefill` reports the window-limited prefill
 in TFLOP/s (64K prompt in 8K chunks at head_dim 128, over bf16 and 8-bit caches,
-and a 32K prompt at head_dim 256); `cpu_baseline` is the fp64 oracle on a
-bounded sample, on the host cores.
+and a 32K prompt at head_dim 256); `append` rates hwkv_append of 8K-token chunks
+against the copy bandwidth; `cpu_baseline` is the fp64 oracle on a bounded sample,
+on the host cores.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
     python bench.py --impl reference ...   # the oracle arm, on host cores
