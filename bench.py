@@ -816,7 +816,6 @@ def main():
         cb = cpu_baseline(wl, r["max_ctx"], r["t_first"] + 1)
     if rank != 0:
         return
-    config["context"] = r["t_end"]
     config["l2"] = ("each timed step preceded by a 2 x L2 read outside its events "
                     "(a layer-step reads less than 2 x L2)" if r["flush"] else
                     "inputs larger than L2 (each layer-step reads more than 2 x 129 MB of K/V)")
@@ -839,6 +838,9 @@ def main():
                      "traffic_source": "ncu dram bytes of a 1-layer batch-2 capture, scaled by "
                                        "algorithmic bytes"},
         "residency_bytes": r["resid_bytes"],
+        "positions": {"t_first_timed": r["t_first"], "t_end": r["t_end"],
+                      "note": "tokens held per row before the first timed step and at the end "
+                              "of the run (config.context is the workload's context)"},
         "e2e": {"value": r["e2e_value"], "unit": "tokens/s", "h2d_bytes_per_step": r["h2d"],
                 "d2h_bytes_per_step": r["d2h"], "steps": r["e2e_steps"]},
         "gpu_launches": r["launches"],

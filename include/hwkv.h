@@ -274,19 +274,31 @@ HWKV_API hwkv_status hwkv_row_len(const hwkv_cache* cache, int32_t layer, int32_
  * Same result and arguments as hwkv_decode_attn, but the partial outputs and
  * the work plan live in a fixed 4 MiB array inside this library's device image
  * (present on every GPU that loads the library until the process exits)
- * instead of the cache's workspace. It calls no cudaMalloc, cudaFree or allocating routine.
+ * instead of the cache's workspace. It calls no cudaMalloc, cudaFree or
+ * allocating routine, and it does not synchronize: the kernels read the
+ * layer's lengths on the device (after graph-mode steps the host copy only
+ * sizes the grid, and the "holds no tokens" check is skipped; rows holding
+ * nothing decode to zeros).
  * The first call on each device, with that device current, looks up the
- * array's device address (cudaGetSymbolAddress); make that first call before
+ * array's device address (cudaGetSymbolAddress) and keeps it for the life of
+ * the process (a device reset is not supported); make that first call before
  * any stream capture. The array keeps the last call's contents and nothing in
  * it needs to start at zero. All calls share it: calls whose kernels overlap
  * on the GPU (other streams, other caches) race and give wrong results.
  * It needs 2 * grid * (32 * head_dim + 64) bytes of partials (grid <= the SM
- * count) plus 16 * (2 + batch * n_kv_heads) bytes of plan, both rounded up to
- * 256: 2.5 MB + 16 B per ring on 152 SMs at head_dim 256. A layout that does
- * not fit fails with HWKV_EINVAL before anything is launched.
+ * count) plus 16 * (2 + batch * n_kv_heads) bytes of plan, each rounded up to
+ * 256 (hwkv_decode_static_scratch_bytes computes it): 2.8 MB on 152 SMs at
+ * head_dim 256 with 256 batch rows and 64 KV heads, the largest valid policy.
+ * A layout that does not fit fails with HWKV_EINVAL before anything is launched.
  */
 HWKV_API hwkv_status hwkv_decode_attn_static(hwkv_cache* cache, int32_t layer, const void* q,
                                              float scale, float* out, void* cuda_stream);
+
+/* Host-only: the static scratch bytes hwkv_decode_attn_static needs for `policy`
+ * on a GPU of num_sms SMs (its largest grid). Returns HWKV_EINVAL (with *bytes
+ * set) when that exceeds HWKV_DECODE_STATIC_SCRATCH_BYTES, as the call would. */
+HWKV_API hwkv_status hwkv_decode_static_scratch_bytes(const hwkv_policy* policy, int32_t num_sms,
+                                                      size_t* bytes);
 
 /*
  * SeqCalib candidate replay (Sec. 3.2: one layer's trace, every candidate
@@ -430,6 +442,17 @@ HWKV_API hwkv_status hwkv_debug_copy_scales(const hwkv_cache* cache, int32_t lay
  * else HWKV_OK.
  */
 HWKV_API hwkv_status hwkv_sync_check(hwkv_cache* cache);
+
+/*
+ * Test of the failure path of every kernel wait (no paper counterpart): launches
+ * one CTA whose thread waits, with the bounded mbarrier wait the kernels use, on
+ * an mbarrier that nothing arrives at; after limit_ns nanoseconds (1e6 .. 2e9)
+ * of the GPU's global timer it gives up and sets the wait-timeout bit of the
+ * cache's error word, exactly as a kernel whose wait ran out would, and ends. No
+ * copy or tensor-core operation is in flight, so the context stays usable; the
+ * next hwkv_sync_check returns HWKV_EKERNEL and clears the word.
+ */
+HWKV_API hwkv_status hwkv_debug_wait_probe(hwkv_cache* cache, int64_t limit_ns, void* cuda_stream);
 
 /* Message of the last failure on this thread ("" if none). */
 HWKV_API const char* hwkv_last_error(void);

@@ -93,6 +93,7 @@ def lib():
             "hwkv_prefill": [_vp, _i32, _vp, _vp, _vp, _i64, ctypes.c_float, _vp, _vp],
             "hwkv_decode_attn": [_vp, _i32, _vp, ctypes.c_float, _vp, _vp],
             "hwkv_decode_attn_static": [_vp, _i32, _vp, ctypes.c_float, _vp, _vp],
+            "hwkv_decode_static_scratch_bytes": [pp, _i32, ctypes.POINTER(ctypes.c_size_t)],
             "hwkv_decode_step": [_vp, _i32, _vp, _vp, _vp, ctypes.c_float, _vp, _vp],
             "hwkv_decode_step_graph": [_vp, _i32, _vp, _vp, _vp, ctypes.c_float, _vp, _vp],
             "hwkv_append_rows": [_vp, _i32, _i32, _i32, _vp, _vp, _i64, _vp],
@@ -108,6 +109,7 @@ def lib():
             "hwkv_debug_copy_ring": [_vp, _i32, _i32, _i32, _vp, _vp],
             "hwkv_debug_copy_scales": [_vp, _i32, _i32, _i32, _vp, _vp],
             "hwkv_sync_check": [_vp],
+            "hwkv_debug_wait_probe": [_vp, _i64, _vp],
             "hwkv_calib_workspace_bytes": [ctypes.POINTER(hwkv_calib_desc),
                                            ctypes.POINTER(ctypes.c_size_t)],
             "hwkv_calib_scores": [ctypes.POINTER(hwkv_calib_desc), _vp, _vp, _vp, ctypes.c_float,
@@ -240,6 +242,13 @@ def hwkv_decode_attn_static(cache, layer, q, scale, out, stream=None):
                                          _stream(stream)))
 
 
+def hwkv_decode_static_scratch_bytes(policy, num_sms):
+    """Static scratch bytes hwkv_decode_attn_static needs (raises HWKV_EINVAL past the array)."""
+    n = ctypes.c_size_t(0)
+    _check(lib().hwkv_decode_static_scratch_bytes(ctypes.byref(policy), num_sms, ctypes.byref(n)))
+    return n.value
+
+
 def hwkv_residency_bytes(cache, layer=-1):
     v = ctypes.c_uint64(0)
     _check(lib().hwkv_residency_bytes(cache, layer, ctypes.byref(v)))
@@ -283,6 +292,10 @@ def hwkv_debug_copy_scales(cache, layer, b, kv_head):
     _check(lib().hwkv_debug_copy_scales(cache, layer, b, kv_head, k.ctypes.data_as(_vp),
                                         v.ctypes.data_as(_vp)))
     return k, v
+
+
+def hwkv_debug_wait_probe(cache, limit_ns, stream=None):
+    _check(lib().hwkv_debug_wait_probe(cache, limit_ns, _stream(stream)))
 
 
 def hwkv_sync_check(cache):

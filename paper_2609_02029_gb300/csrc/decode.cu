@@ -961,6 +961,25 @@ cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cuda
   }
 }
 
+// The bounded wait on its own: thread 0 waits for phase 0 of a freshly initialised
+// mbarrier that no thread and no copy will ever arrive at, so the wait runs out after
+// limit_ns and sets kErrWaitTimeout, as a kernel wait that gives up would. Nothing
+// asynchronous is in flight and nothing else waits, so the CTA then simply ends.
+__global__ void wait_probe_kernel(int* err, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait_bounded(&bar, 0u, err, limit_ns);
+}
+
+cudaError_t launch_wait_probe(int* err, uint64_t limit_ns, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(err, limit_ns);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s) {
   const dim3 grid(p.batch * p.n_q_heads), block(kCombineWarps * 32);
   switch (head_dim) {

@@ -173,6 +173,8 @@ cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtens
                               const CUtensorMap& ck_map, const CUtensorMap& cv_map,
                               const CUtensorMap& ring_map, cudaStream_t s, bool fp8 = false);
 int decode_smem_bytes(int head_dim);
+// one CTA waiting, with the kernels' bounded wait, on an mbarrier nothing arrives at
+cudaError_t launch_wait_probe(int* err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t decode_prepare_device();  // one-time kernel attributes on the current device
 
 // ------------------------------------------------------------ device PTX
@@ -247,14 +249,17 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
-// Waits for the phase of `parity` to complete, giving up after ~2 s.
-// Returns false (and sets the error word) on timeout.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, int* err) {
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // every kernel wait gives up after 2 s
+
+// Waits for the phase of `parity` to complete, giving up after limit_ns of
+// %globaltimer. Returns false (and sets the error word) on timeout.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, int* err,
+                                                  uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0u && globaltimer_ns() - t0 > 2000000000ull) {
+    if ((i & 255u) == 0u && globaltimer_ns() - t0 > limit_ns) {
       atomicOr(err, kErrWaitTimeout);
       return false;
     }

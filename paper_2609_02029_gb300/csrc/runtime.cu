@@ -807,6 +807,15 @@ hwkv_status hwkv_sync_check(hwkv_cache* c) {
   return ok();
 }
 
+hwkv_status hwkv_debug_wait_probe(hwkv_cache* c, int64_t limit_ns, void* cuda_stream) {
+  if (!c) return fail(HWKV_EINVAL, "cache is NULL");
+  if (limit_ns < 1000000 || limit_ns > 2000000000)
+    return fail(HWKV_EINVAL, "limit_ns %lld outside [1e6, 2e9]", (long long)limit_ns);
+  cudaError_t e = launch_wait_probe(c->err(), (uint64_t)limit_ns, static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return fail(HWKV_ECUDA, "wait probe launch: %s", cudaGetErrorString(e));
+  return ok();
+}
+
 // ---------------------------------------------------------------------------
 // Decode without any device allocation. Some callers cannot allocate device
 // memory at all: code embedded in another engine whose allocator owns every
@@ -827,6 +836,37 @@ hwkv_status hwkv_sync_check(hwkv_cache* c) {
 // streams, or two caches, at once) race on it.
 static __device__ __align__(256) uint8_t g_decode_static_scratch[HWKV_DECODE_STATIC_SCRATCH_BYTES];
 
+// Byte layout of the static scratch for a decode launch of `grid` CTAs: two
+// partial slots per CTA (outputs, then (max, sum) pairs), then the plan table.
+struct StaticScratch {
+  size_t o_bytes, ml_bytes, plan_bytes;
+  size_t total() const { return o_bytes + ml_bytes + plan_bytes; }
+};
+static StaticScratch static_scratch_layout(int grid, int head_dim, int batch, int n_kv_heads) {
+  StaticScratch s;
+  s.o_bytes = align_up((size_t)2 * grid * kMaxGroup * head_dim * 4, kAlign);
+  s.ml_bytes = align_up((size_t)2 * grid * kMaxGroup * 8, kAlign);
+  s.plan_bytes = align_up((size_t)(4 + 2 * (size_t)batch * n_kv_heads) * 8, kAlign);
+  return s;
+}
+
+hwkv_status hwkv_decode_static_scratch_bytes(const hwkv_policy* policy, int32_t num_sms,
+                                             size_t* bytes) {
+  if (!bytes) return fail(HWKV_EINVAL, "bytes is NULL");
+  hwkv_status st = validate(policy);
+  if (st != HWKV_OK) return st;
+  if (num_sms <= 0) return fail(HWKV_EINVAL, "num_sms must be positive");
+  const StaticScratch s =
+      static_scratch_layout(num_sms, policy->head_dim, policy->batch, policy->n_kv_heads);
+  *bytes = s.total();
+  if (s.total() > HWKV_DECODE_STATIC_SCRATCH_BYTES)
+    return fail(HWKV_EINVAL, "static decode needs %zu scratch bytes > %u", s.total(),
+                (unsigned)HWKV_DECODE_STATIC_SCRATCH_BYTES);
+  return ok();
+}
+
+// The array's device address per device ordinal, looked up once and kept for
+// the life of the process (a device reset would leave it stale; not supported).
 static void* static_scratch_address(int device, cudaError_t* err) {
   constexpr int kMaxDevices = 64;
   static std::mutex mu;
@@ -848,21 +888,23 @@ static void* static_scratch_address(int device, cudaError_t* err) {
 
 hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q, float scale,
                                     float* out, void* cuda_stream) {
-  hwkv_status st = check_fresh(c, layer);
+  // no length refresh here: that would synchronize the device. The kernels plan
+  // from the device lengths; the host copy only sizes the grid (an estimate when
+  // graph-mode steps own the layer), and rows holding nothing decode to zeros.
+  hwkv_status st = check_layer(c, layer);
   if (st != HWKV_OK) return st;
   if (!q || !out) return fail(HWKV_EINVAL, "q/out is NULL");
   if (!(scale > 0.f) || scale == INFINITY) return fail(HWKV_EINVAL, "scale must be positive and finite");
-  bool any = false;
-  for (int b = 0; b < c->pol.batch; ++b) any |= c->row_t(layer, b) > 0;
-  if (!any) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
+  if (!c->dev_owned[layer]) {
+    bool any = false;
+    for (int b = 0; b < c->pol.batch; ++b) any |= c->row_t(layer, b) > 0;
+    if (!any) return fail(HWKV_EINVAL, "layer %d holds no tokens", layer);
+  }
   const int d = c->pol.head_dim;
   const int grid = decode_grid_cap(c, step_tokens(c, layer, 0));
-  // two partial slots per CTA, then the plan table
-  const size_t o_bytes = align_up((size_t)2 * grid * kMaxGroup * d * 4, kAlign);
-  const size_t ml_bytes = align_up((size_t)2 * grid * kMaxGroup * 8, kAlign);
-  const size_t plan_bytes = (size_t)(4 + 2 * c->pol.batch * c->pol.n_kv_heads) * 8;
-  if (o_bytes + ml_bytes + plan_bytes > HWKV_DECODE_STATIC_SCRATCH_BYTES)
-    return fail(HWKV_EINVAL, "static decode needs %zu scratch bytes > %u", o_bytes + ml_bytes + plan_bytes,
+  const StaticScratch sl = static_scratch_layout(grid, d, c->pol.batch, c->pol.n_kv_heads);
+  if (sl.total() > HWKV_DECODE_STATIC_SCRATCH_BYTES)
+    return fail(HWKV_EINVAL, "static decode needs %zu scratch bytes > %u", sl.total(),
                 (unsigned)HWKV_DECODE_STATIC_SCRATCH_BYTES);
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -876,8 +918,8 @@ hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q,
   p.scale_log2 = scale * 1.4426950408889634f;
   p.q = static_cast<const __nv_bfloat16*>(q);
   p.part_o = reinterpret_cast<float*>(scratch);
-  p.part_ml = reinterpret_cast<float2*>(scratch + o_bytes);
-  p.plan = reinterpret_cast<int64_t*>(scratch + o_bytes + ml_bytes);
+  p.part_ml = reinterpret_cast<float2*>(scratch + sl.o_bytes);
+  p.plan = reinterpret_cast<int64_t*>(scratch + sl.o_bytes + sl.ml_bytes);
   p.out = out;
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   e = launch_decode(p, c->kv_map, c->kv_map, d, grid, s, c->fp8());

@@ -53,3 +53,50 @@ def test_null_arguments_rejected_without_device():
     with pytest.raises(hwkv.HwkvError):
         hwkv.hwkv_residency_bytes(None)
     hwkv.hwkv_free(None)
+
+
+def test_arena_smaller_than_required_is_enomem_before_any_device_call():
+    """hwkv_alloc checks a caller-owned arena's size before touching the device:
+    one byte short of hwkv_required_bytes gives HWKV_ENOMEM (the pointer is never
+    dereferenced, so a made-up aligned address is enough here)."""
+    pol = hwkv.make_policy(2, 2, 8, 128, 3, 5000, [0, 100, 4096, 0])
+    need = hwkv.hwkv_required_bytes(pol)
+    fake_arena = 1 << 40  # 256-byte aligned, never touched
+    for short in (need - 1, need // 2, 0):
+        with pytest.raises(hwkv.HwkvError) as e:
+            hwkv.hwkv_alloc(pol, fake_arena, short, 0)
+        assert e.value.status == hwkv.HWKV_ENOMEM
+        assert "required" in hwkv.hwkv_last_error()
+
+
+def _static_need(grid, d, batch, hkv):
+    """The size rule written out independently: two partial slots per CTA of
+    kMaxGroup (8) query heads x d fp32 outputs, then 8 (max, sum) pairs of fp32,
+    then the int64 plan table (4 + 2 per ring), each rounded up to 256 bytes."""
+    up = lambda x: (x + 255) // 256 * 256
+    return up(2 * grid * 8 * d * 4) + up(2 * grid * 8 * 8) + up((4 + 2 * batch * hkv) * 8)
+
+
+@pytest.mark.parametrize("sms,batch,hkv,d", [
+    (152, 256, 64, 256),   # the largest valid policy on this GPU's SM count
+    (160, 256, 64, 256),   # a few more SMs still fit
+    (148, 1, 1, 64),
+    (152, 16, 4, 128),
+])
+def test_static_decode_scratch_fits(sms, batch, hkv, d):
+    pol = hwkv.make_policy(1, hkv, hkv * 8, d, batch, 1000, [0] * hkv)
+    got = hwkv.hwkv_decode_static_scratch_bytes(pol, sms)
+    assert got == _static_need(sms, d, batch, hkv)
+    assert got <= 4 << 20
+
+
+def test_static_decode_scratch_too_small_is_einval():
+    # 256 SMs (the decode's slot limit) at head_dim 256 and the largest plan: > 4 MiB
+    pol = hwkv.make_policy(1, 64, 512, 256, 256, 1000, [0] * 64)
+    with pytest.raises(hwkv.HwkvError) as e:
+        hwkv.hwkv_decode_static_scratch_bytes(pol, 256)
+    assert e.value.status == hwkv.HWKV_EINVAL
+    assert _static_need(256, 256, 256, 64) > 4 << 20
+    with pytest.raises(hwkv.HwkvError) as e:
+        hwkv.hwkv_decode_static_scratch_bytes(pol, 0)
+    assert e.value.status == hwkv.HWKV_EINVAL

@@ -189,3 +189,35 @@ def test_library_allocated_arena():
         assert hwkv.hwkv_residency_bytes(c) == 0
     finally:
         hwkv.hwkv_free(c)
+
+
+def test_bounded_wait_gives_up_and_reports():
+    """The kernels' bounded mbarrier wait, run out on purpose (an mbarrier nothing
+    arrives at, a 50 ms limit, nothing asynchronous in flight): the error word
+    reaches the host as HWKV_EKERNEL, the word is cleared, and the cache and the
+    context keep working."""
+    import time
+    import torch
+    r = Run(1, 1, 8, 2, 64, 400, [0, 128], seed=1)
+    try:
+        r.fill(0, 200)
+        hwkv.hwkv_sync_check(r.cache)
+        t0 = time.perf_counter()
+        hwkv.hwkv_debug_wait_probe(r.cache, 50_000_000, r.stream)
+        with pytest.raises(hwkv.HwkvError) as e:
+            hwkv.hwkv_sync_check(r.cache)
+        assert e.value.status == hwkv.HWKV_EKERNEL
+        assert "0x1" in str(e.value)
+        assert time.perf_counter() - t0 >= 0.05
+        hwkv.hwkv_sync_check(r.cache)  # cleared
+        out = r.decode_step(0).cpu().numpy()
+        p = hwkv.hwkv_seq_len(r.cache, 0) - 1
+        for qh in range(8):
+            assert_close(out[0, qh], r.oracle_rows(0, 0, qh, [p])[0], "decode after the probe")
+        hwkv.hwkv_sync_check(r.cache)
+        with pytest.raises(hwkv.HwkvError) as e:
+            hwkv.hwkv_debug_wait_probe(r.cache, 10, r.stream)  # below the 1 ms floor
+        assert e.value.status == hwkv.HWKV_EINVAL
+        torch.cuda.synchronize()
+    finally:
+        r.close()

@@ -53,27 +53,61 @@ def test_prompt_then_every_decode_output(name):
         r.close()
 
 
-def test_prefill64k_sampled_rows():
+def test_prefill64k_rows():
+    """prefill64k (64K prompt in 8 chunks of 8,192, batch 2, 32q/8kv, head_dim 128):
+    every row of chunk 0 for every (batch row, query head); on each later chunk
+    the rows within 2 of the chunk's first and last position and of each window
+    edge, plus 512 seeded random rows per (batch row, query head). The oracle runs
+    over host arrays of each KV head's whole history (generated once), one oracle
+    thread per worker, while the GPU continues."""
+    import os
+    import threading
+    from concurrent.futures import ThreadPoolExecutor
+
+    import hwkv_gen
+    import oracle
     wl = workloads.make("prefill64k")
     r = Run.for_workload(wl)
     rng = np.random.default_rng(1)
+    B, Hq, Hkv, d, G, n = wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.group, wl.chunk
+    K = [[hwkv_gen.fill_host_sub(r.g, hwkv_gen.K, 0, b, 0, wl.prompt, h, 1, d)[:, 0]
+          for h in range(Hkv)] for b in range(B)]
+    V = [[hwkv_gen.fill_host_sub(r.g, hwkv_gen.V, 0, b, 0, wl.prompt, h, 1, d)[:, 0]
+          for h in range(Hkv)] for b in range(B)]
+    local = threading.local()
+
+    def check(b, qh, rows, t0, got, Q):
+        if not getattr(local, "set", False):
+            oracle.set_threads(1)
+            local.set = True
+        h = qh // G
+        pos = [t0 + i for i in rows]
+        want, sp = oracle.window_attention_bf16(Q, pos, K[b][h], V[b][h], r.window(0, h), r.scale)
+        np.testing.assert_allclose(sp, 1.0, atol=1e-12)
+        assert_close(got, want, "prefill64k b%d q%d chunk@%d (%d rows)" % (b, qh, t0, len(rows)))
+
+    ex = ThreadPoolExecutor(max_workers=os.cpu_count() or 1)
+    futures = []
     try:
         done = 0
         while done < wl.prompt:
-            n = wl.chunk
             out = r.prefill(0, n).cpu().numpy()
-            rows = _prefill_rows(n, done, wl.windows, rng, k=8) if done else list(range(0, n, 61))
-            for b in range(wl.batch):
-                heads = [int(x) for x in rng.choice(wl.n_q_heads, size=6, replace=False)]
-                for qh in heads:
-                    # chunk 0: every row for two of the sampled heads
-                    rr = list(range(n)) if (done == 0 and qh in heads[:2]) else rows
-                    assert_close(out[b, rr, qh],
-                                 r.oracle_rows(0, b, qh, [done + i for i in rr]),
-                                 "prefill64k b%d q%d chunk@%d" % (b, qh, done))
+            Qc = hwkv_gen.fill_host(r.g, hwkv_gen.Q, 0, B, done, n, Hq, d)
+            edges = _prefill_rows(n, done, wl.windows, rng, k=0)
+            for b in range(B):
+                for qh in range(Hq):
+                    if done == 0:
+                        rows = list(range(n))
+                    else:
+                        rows = sorted(set(edges) | set(rng.choice(n, size=512, replace=False).tolist()))
+                    futures.append(ex.submit(check, b, qh, rows, done, out[b, rows, qh].copy(),
+                                             Qc[b, rows, qh].copy()))
             done += n
         r.check_rings(0)
         r.check_residency()
         hwkv.hwkv_sync_check(r.cache)
+        for f in futures:
+            f.result()
     finally:
+        ex.shutdown(wait=True, cancel_futures=True)
         r.close()
