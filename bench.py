@@ -41,6 +41,10 @@ L2_BYTES = 129 * 1024 * 1024
 # traffic is reads of every resident K/V row plus tile partials, so it scales with the
 # algorithmic bytes of a launch. Set to None whenever that kernel changes.
 DECODE_TRAFFIC_PER_BYTE = (244.301312e6 + 3.917312e6) / 244066304.0
+# tensor-pipe activity of the prefill kernel (ncu sm__pipe_tensor_cycles_active, pct of peak
+# sustained active) from the one-launch --set full capture summarised in the named profile;
+# set to None whenever that kernel changes.
+PREFILL_TENSOR_PIPE = {"prefill64k": (0.507, "profiles/prefill_tc_prefill64k_full.md")}
 
 
 def peaks():
@@ -412,6 +416,39 @@ def run_gpu(args, wl, world, rank, local, fp8=False):
                 graph_value=graph_value, graph_ms=graph_ms, graph_steps=graph_steps)
 
 
+SECONDARY_WORKLOADS = ["tiny", "single32k", "budget161k_r25", "budget161k_r50",
+                       "budget161k_r75", "budget161k_r100"]
+
+
+def workload_by_name(name):
+    if name.startswith("budget161k_r"):
+        return workloads.make("budget161k", int(name.split("_r")[1]) / 100.0)
+    return workloads.make(name)
+
+
+def run_secondary(args, name, world, rank, local, hbm):
+    """The same decode step on another workload (fewer timed steps): device-timed
+    tokens/s, the replayed-graph form, end to end, and the decode call's rate
+    against the copy bandwidth."""
+    wl = workload_by_name(name)
+    a = argparse.Namespace(**vars(args))
+    a.steps, a.e2e_steps = min(args.steps, 32), min(args.e2e_steps, 8)
+    r = run_gpu(a, wl, world, rank, local)
+    return {"workload": wl.name, "layers": wl.n_layers, "batch_per_gpu": wl.batch,
+            "head_dim": wl.head_dim, "context": wl.max_ctx, "windows": wl.note,
+            "value": r["value"], "unit": "tokens/s", "steps": a.steps,
+            "ms_per_step": r["ms"] / a.steps,
+            "graph_value": r["graph_value"], "graph_ms_per_step": r["graph_ms"] / r["graph_steps"],
+            "e2e_value": r["e2e_value"],
+            "decode_gbs": r["achieved_gbs"], "frac": r["achieved_gbs"] / hbm,
+            "bytes_per_launch": r["bytes_avg"], "launch_ms": r["dec_avg_ms"],
+            "step_bytes": r["step_bytes"],
+            "graph_step_gbs": r["step_bytes"] / (r["graph_ms"] / r["graph_steps"] * 1e-3) / 1e9,
+            "l2": ("each timed step preceded by a 2 x L2 read outside its events"
+                   if r["flush"] else "inputs larger than L2"),
+            "residency_bytes": r["resid_bytes"]}
+
+
 # ------------------------------------------------------------- GPU prefill
 def prefill_flops(wl, t0, n):
     """Algorithmic flops of one prefill chunk: 4 d G per visible (query, key) pair."""
@@ -487,14 +524,16 @@ def run_prefill(args, local, fp8=False, workload="prefill64k"):
 
 
 # ------------------------------------------------------------ GPU append
-def run_append(local, n=8192, reps=10, warm=3):
+def run_append(local, n=8192, reps=10, warm=3, fp8=False):
     """hwkv_append of 8,192-token chunks into layer 0 of layers16_112k (batch 16,
     4 KV heads, d 256, rings of {full, 32768, 8192, 2048, 512} drawn per head):
     each call reads the chunk's K and V (537 MB, more than L2) and writes the last
     min(n, cap) tokens of every head into its ring. Algorithmic bytes per call:
     batch x sum_h min(n, cap_h) x 4d written plus the same read from the input
     (only the rows that land are read). Full heads hold max_ctx = 14 chunks, so at
-    most 14 calls."""
+    most 14 calls. With fp8 the cache holds E4M3 codes + one fp32 scale per row: bytes
+    per landing row and head are the bf16 K and V read (4d) plus codes and scales
+    written (2d + 8)."""
     import torch
 
     import hwkv_gen
@@ -511,12 +550,14 @@ def run_append(local, n=8192, reps=10, warm=3):
     v = torch.empty_like(k)
     hwkv_gen.fill_device(g, hwkv_gen.K, 0, B, 0, n, Hkv, d, k.data_ptr(), s)
     hwkv_gen.fill_device(g, hwkv_gen.V, 0, B, 0, n, Hkv, d, v.data_ptr(), s)
-    pol = hwkv.make_policy(1, Hkv, wl.n_q_heads, d, B, wl.max_ctx, windows)
+    pol = hwkv.make_policy(1, Hkv, wl.n_q_heads, d, B, wl.max_ctx, windows,
+                           kv_format=hwkv.HWKV_KV_FP8_E4M3 if fp8 else hwkv.HWKV_KV_BF16)
     nbytes = hwkv.hwkv_required_bytes(pol)
     arena = torch.empty(nbytes, dtype=torch.uint8, device=dev)
     cache = hwkv.hwkv_alloc(pol, arena, nbytes, s)
     caps = [wl.max_ctx if (W == 0 or W >= wl.max_ctx) else W for W in windows]
-    per_call = 2 * B * sum(min(n, c) for c in caps) * 4 * d
+    per_row = (4 * d + 2 * d + 8) if fp8 else 2 * 4 * d
+    per_call = B * sum(min(n, c) for c in caps) * per_row
     times = []
     for i in range(warm + reps):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -531,7 +572,8 @@ def run_append(local, n=8192, reps=10, warm=3):
     ms = float(np.median(times))
     del k, v, arena
     torch.cuda.empty_cache()
-    return {"workload": "layers16_112k layer 0, 8192-token chunks", "ms": ms,
+    return {"workload": "layers16_112k layer 0, 8192-token chunks" + (", 8-bit cache" if fp8 else ""),
+            "ms": ms,
             "bytes_per_call": per_call, "gbs": per_call / (ms * 1e-3) / 1e9}
 
 
@@ -598,99 +640,91 @@ def step_keys(wl, max_ctx, t):
     return out
 
 
-class OracleSample:
-    """A bounded sample of one decode step for the fp64 oracle (array form):
-    units drawn at random, their q/K/V generated on the host before any clock
-    starts, at most `max_bytes` of inputs held."""
+class OracleLayerSteps:
+    """The fp64 oracle (array form) over whole layer-steps of the decode: for one
+    layer at position p, every (batch row, KV head) unit's G queries over all of
+    its retained keys. A layer's inputs are generated on the host before its clock
+    starts (one unit per thread); then the oracle runs over every unit of the layer
+    with all host cores busy (one unit per thread, one OpenMP thread each), largest
+    units first, and only that is timed."""
 
-    def __init__(self, wl, max_ctx, t, max_units, max_bytes=3 << 30, seed=12345):
+    def __init__(self, wl, max_ctx):
+        self.wl, self.max_ctx = wl, max_ctx
+        self.cores = os.cpu_count() or 1
+        self.units_per_layer = wl.batch * wl.n_kv_heads
+
+    def _inputs(self, layer, p):
         from concurrent.futures import ThreadPoolExecutor
 
         import hwkv_gen
         import oracle
 
-        self.wl, self.t = wl, t
-        self.cores = os.cpu_count() or 1
-        self.units_all = step_keys(wl, max_ctx, t)
-        self.keys_all = sum(u[4] for u in self.units_all)
+        wl = self.wl
         g = hwkv_gen.desc(wl.seed, wl.per_head_scale)
-        d, G, p = wl.head_dim, wl.group, t - 1
-        rng = np.random.default_rng(seed)
-        order = rng.permutation(len(self.units_all))
-        chosen, held = [], 0
-        for i in order[:max_units]:
-            u = self.units_all[i]
-            nb = u[4] * d * 2 * 2
-            if chosen and held + nb > max_bytes:
-                break
-            chosen.append(u)
-            held += nb
+        d, G = wl.head_dim, wl.group
+        units = []
+        for h in range(wl.n_kv_heads):
+            W = wl.windows[layer * wl.n_kv_heads + h]
+            Weff = 0 if (W == 0 or W >= self.max_ctx) else W
+            for b in range(wl.batch):
+                units.append((b, h, Weff))
 
         def make(u):
-            l, b, h, W, n = u
+            b, h, W = u
             lo = oracle.window_lo(p, W)
-            K = hwkv_gen.fill_host_sub(g, hwkv_gen.K, l, b, lo, p - lo + 1, h, 1, d)[:, 0]
-            V = hwkv_gen.fill_host_sub(g, hwkv_gen.V, l, b, lo, p - lo + 1, h, 1, d)[:, 0]
-            Q = hwkv_gen.fill_host_sub(g, hwkv_gen.Q, l, b, p, 1, h * G, G, d)[0]
+            K = hwkv_gen.fill_host_sub(g, hwkv_gen.K, layer, b, lo, p - lo + 1, h, 1, d)[:, 0]
+            V = hwkv_gen.fill_host_sub(g, hwkv_gen.V, layer, b, lo, p - lo + 1, h, 1, d)[:, 0]
+            Q = hwkv_gen.fill_host_sub(g, hwkv_gen.Q, layer, b, p, 1, h * G, G, d)[0]
             return (Q, K, V, p - lo)
 
         with ThreadPoolExecutor(max_workers=self.cores) as ex:
-            self.inputs = list(ex.map(make, chosen))
-        self.keys = [x[1].shape[0] for x in self.inputs]
+            inputs = list(ex.map(make, units))
+        inputs.sort(key=lambda x: -x[1].shape[0])
+        return inputs
 
-    def run(self, n_units=None):
-        """Seconds the oracle takes on the first n_units sampled units, all host
-        cores busy (one unit per thread, one OpenMP thread each)."""
+    def run_layer(self, layer, p):
+        """(seconds, units, keys) of the oracle over every unit of `layer` at position p."""
         import threading
         from concurrent.futures import ThreadPoolExecutor
 
         import oracle
 
-        units = self.inputs[:n_units] if n_units else self.inputs
+        inputs = self._inputs(layer, p)
         local = threading.local()
-        d = self.wl.head_dim
+        gamma = 1.0 / np.sqrt(self.wl.head_dim)
 
         def work(u):
             if not getattr(local, "set", False):
                 oracle.set_threads(1)
                 local.set = True
             Q, K, V, p_rel = u
-            oracle.window_attention_bf16(Q, [p_rel] * len(Q), K, V, 0, 1.0 / np.sqrt(d))
+            oracle.window_attention_bf16(Q, [p_rel] * len(Q), K, V, 0, gamma)
 
-        t0 = time.perf_counter()
         with ThreadPoolExecutor(max_workers=self.cores) as ex:
-            list(ex.map(work, units))
-        return time.perf_counter() - t0, len(units), sum(self.keys[:len(units)])
-
-    def step_seconds(self, sec, keys):
-        """Whole-step time, scaling the sample by keys attended (cost is linear in keys)."""
-        return sec * self.keys_all / max(keys, 1)
-
-    def describe(self, n, keys, sec, passes=1):
-        rep = " (mean of %d passes)" % passes if passes > 1 else ""
-        return ("%d of %d (layer, batch row, KV head) units of one decode step at t=%d, "
-                "%d of %d keys, fp64 oracle %.2f s%s on %d threads, scaled by keys to the full "
-                "step" % (n, len(self.units_all), self.t, keys, self.keys_all, sec, rep,
-                          self.cores))
+            t0 = time.perf_counter()
+            list(ex.map(work, inputs))
+            sec = time.perf_counter() - t0
+        return sec, len(inputs), sum(x[1].shape[0] for x in inputs)
 
 
-def cpu_baseline(wl, max_ctx, t, budget_s=15.0, min_s=10.0):
-    """Oracle tokens/s on this host's cores from a bounded sample of one step: the
-    sampled units are run again until about `min_s` seconds of oracle work are timed."""
-    cores = os.cpu_count() or 1
-    samp = OracleSample(wl, max_ctx, t, max_units=8 * cores)
-    sec, n, keys = samp.run()
-    if sec > budget_s and n > cores:  # keep the timed work bounded
-        m = max(cores, int(n * budget_s / sec))
-        sec, n, keys = samp.run(m)
-    total, passes = sec, 1
-    while total < min_s and passes < 64:
-        total += samp.run(n)[0]
-        passes += 1
-    sec = total / passes
-    step_s = samp.step_seconds(sec, keys)
-    return {"value": wl.batch / step_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": samp.describe(n, keys, sec, passes)}
+def cpu_baseline(wl, max_ctx, t, steps=2):
+    """Oracle tokens/s on this host's cores over `steps` whole decode steps (every
+    layer, batch row and KV head) at positions t - 1, t, ...; input generation is
+    outside the timed part."""
+    orc = OracleLayerSteps(wl, max_ctx)
+    sec, units, keys = 0.0, 0, 0
+    for st in range(steps):
+        for layer in range(wl.n_layers):
+            s_, u_, k_ = orc.run_layer(layer, t - 1 + st)
+            sec += s_
+            units += u_
+            keys += k_
+    return {"value": wl.batch * steps / sec, "unit": "tokens/s", "cores": orc.cores,
+            "kind": "oracle", "seconds": sec,
+            "sample": "%d whole decode steps at t=%d..%d: all %d (layer, batch row, KV head) "
+                      "units each, %d keys in all; fp64 oracle %.1f s on %d threads (input "
+                      "generation before each layer's clock, not timed)"
+                      % (steps, t, t + steps - 1, units // steps, keys, sec, orc.cores)}
 
 
 # ------------------------------------------------------------------ main
@@ -716,6 +750,9 @@ def main():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-calib", action="store_true")
+    ap.add_argument("--no-secondary", action="store_true",
+                    help="skip the decode lines of the other workloads (tiny, single32k, the "
+                         "161K budget sweep)")
     ap.add_argument("--prefill-only", action="store_true",
                     help="run only a prefill measurement (profiling)")
     ap.add_argument("--append-only", action="store_true",
@@ -753,32 +790,43 @@ def main():
     if args.impl == "reference":
         if rank != 0:
             return
-        max_ctx = wl.max_ctx
-        t = wl.prompt + 1
-        cores = os.cpu_count() or 1
-        samp = OracleSample(wl, max_ctx, t, max_units=4 * cores)
-        budget = max(0.5, 120.0 / (args.steps + args.warmup))  # whole run within minutes
-        sec, n, keys = samp.run()
-        m = n if sec <= budget else max(1, int(n * budget / sec))
-        times = []
+        # each step = the decode of `lps` layers (all batch rows and KV heads) by the fp64
+        # oracle on the host cores: lps / L of a whole decode step, so the steps cover
+        # whole decode steps (L / lps steps each) at advancing positions
+        lps = max(1, wl.n_layers // 8)
+        orc = OracleLayerSteps(wl, wl.max_ctx)
+        times, keys = [], 0
         for i in range(args.warmup + args.steps):
-            sec, n, keys = samp.run(m)
+            sec = 0.0
+            for k in range(lps):
+                j = i * lps + k
+                layer, p = j % wl.n_layers, wl.prompt + j // wl.n_layers
+                s_, _, k_ = orc.run_layer(layer, p)
+                sec += s_
+                if i >= args.warmup:
+                    keys += k_
             if i >= args.warmup:
-                times.append(samp.step_seconds(sec, keys))
+                times.append(sec)
         step_s = float(np.mean(times))
-        v = wl.batch / step_s
+        v = wl.batch * lps / wl.n_layers / step_s
+        sample = ("each step: the oracle over every (batch row, KV head) unit of %d of the %d "
+                  "layers (%d units), layers in turn, positions advancing by one per %d steps; "
+                  "%d keys over the %d timed steps; fp64 on %d threads (input generation "
+                  "outside the clock)" % (lps, wl.n_layers, lps * orc.units_per_layer,
+                                          wl.n_layers // lps, keys, args.steps, orc.cores))
         emit({"metric": metric, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
               "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
               "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
               "data": "synthetic", "config": config, "impl": "reference",
-              "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                               "sample": samp.describe(n, keys, sec) + "; each step"},
+              "step_fraction_of_decode_step": lps / wl.n_layers,
+              "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": orc.cores,
+                               "kind": "oracle", "sample": sample},
               "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                       "d2h_bytes_per_step": 0}})
         return
 
     if args.append_only:
-        a = run_append(local)
+        a = run_append(local, fp8=args.kv == "fp8")
         emit({"metric": "append GB/s", "value": a["gbs"], "unit": "GB/s", "n_gpus": 1,
               "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
               "config": {"workload": a["workload"]}, "ms": a["ms"],
@@ -808,6 +856,12 @@ def main():
             pre8 = run_prefill(args, local, fp8=True)
         pre256 = run_prefill(args, local, workload="single32k")
     app = run_append(local) if (not args.no_prefill and rank == 0) else None
+    app8 = run_append(local, fp8=True) if (app is not None and not args.no_fp8) else None
+    sec_lines = None
+    if not args.no_secondary and args.kv == "bf16" and not (args.layers or args.batch):
+        sec_lines = {}
+        for name in SECONDARY_WORKLOADS:
+            sec_lines[name] = run_secondary(args, name, world, rank, local, hbm)
     cal = None
     if rank == 0 and not args.no_calib:
         cal = run_calib(local)
@@ -865,6 +919,10 @@ def main():
                            "frac_of_sustained": pre["tflops"] / tf_sust,
                            "peak_source": peak_src, "ms": pre["ms"],
                            "tokens_per_s": pre["tokens_per_s"], "flops": pre["flops"]}
+        tp = PREFILL_TENSOR_PIPE.get("prefill64k")
+        if tp is not None:
+            line["prefill"]["tensor_pipe_active_ncu"] = tp[0]
+            line["prefill"]["tensor_pipe_source"] = tp[1]
         if pre8 is not None:
             line["prefill"]["fp8_kv"] = {
                 "tflops": pre8["tflops"], "ms": pre8["ms"], "tokens_per_s": pre8["tokens_per_s"],
@@ -882,6 +940,13 @@ def main():
                           "ms": app["ms"], "bytes_per_call": app["bytes_per_call"],
                           "note": "hwkv_append alone (the decode step fuses its one-token append); "
                                   "bytes = rows written + the same rows read"}
+        if app8 is not None:
+            line["append"]["fp8_kv"] = {
+                "gbs": app8["gbs"], "frac": app8["gbs"] / hbm, "ms": app8["ms"],
+                "bytes_per_call": app8["bytes_per_call"],
+                "note": "8-bit cache: bf16 K/V read, E4M3 codes + fp32 row scales written"}
+    if sec_lines is not None:
+        line["other_workloads"] = sec_lines
     if cal is not None:
         line["seqcalib"] = cal
     if cb is not None:

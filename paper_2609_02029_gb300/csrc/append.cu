@@ -9,6 +9,8 @@
 // rows' new lengths in the device length array. One launch covers every KV head
 // and batch row of a layer (grid y and z); each thread moves 16-byte vectors of the
 // rows that land, reads coalesced within each input row and writes over the ring rows.
+#include <algorithm>
+
 #include "hwkv_internal.cuh"
 
 namespace hwkv {
@@ -54,48 +56,61 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
   }
 }
 
-// The 8-bit format (E4M3 codes, one fp32 scale per stored row): one warp per
-// (batch row, token, KV head) row, each lane D/32 consecutive channels.
+// The 8-bit format (E4M3 codes, one fp32 scale per stored row), laid out as the
+// bf16 kernel: block (x, h, b) takes the landing tokens of KV head h of batch row
+// b, one warp per token row (K and V), each lane D/32 consecutive channels.
 // amax = max |x|; s = amax / 448 (IEEE division); code = E4M3 of x / s (IEEE
 // division, round to nearest even, saturating); amax = 0 stores s = 0 and zeros.
 template <int D>
 __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   constexpr int PER = D / 32;
   grid_dep_wait();
-  if (blockIdx.x == 0 && p.lens != nullptr)
+  if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && p.lens != nullptr)
     for (int b = threadIdx.x; b < p.batch; b += blockDim.x)
       p.lens[p.row0 + b] = (int32_t)(p.t0[b] + p.n);
+  const int h = blockIdx.y, b = blockIdx.z;
   const int lane = threadIdx.x & 31;
-  const int64_t total = (int64_t)p.batch * p.n * p.n_units;
-  const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
-  for (int64_t e = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); e < total;
-       e += warps) {
-    const int h = (int)(e % p.n_units);
-    const int64_t r = e / p.n_units;
-    const int64_t i = r % p.n;
-    const int b = (int)(r / p.n);
-    const AppendUnit& u = p.u[h];
-    const int64_t pos = (int64_t)p.t0[b] + i;
-    if (pos >= u.sink && pos < (int64_t)p.t0[b] + p.n - (u.cap - u.sink)) continue;
-    const int64_t slot = ring_slot(pos, u.cap, u.sink);
-    const int64_t src = ((((int64_t)b * p.n + i) * p.n_units + h) * D) + lane * PER;
-    const int64_t rows[2] = {u.k_row0 + (int64_t)(p.row0 + b) * u.stride + slot,
-                             u.v_row0 + (int64_t)(p.row0 + b) * u.stride + slot};
+  const AppendUnit& u = p.u[h];
+  const int64_t n = p.n, t0 = p.t0[b];
+  const int64_t wr = u.cap - u.sink;
+  const int64_t ns = u.sink - t0 <= 0 ? 0 : (u.sink - t0 < n ? u.sink - t0 : n);
+  const int64_t iw = n - wr > ns ? n - wr : ns;  // first new token kept in the window region
+  const int64_t count = ns + (n - iw);
+  const int64_t base = iw < n ? (t0 + iw - u.sink) % wr : 0;  // window slot of token iw
+  const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;
+  const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.stride;
+  const int64_t wstride = (int64_t)gridDim.x * (blockDim.x / 32);
+  for (int64_t j = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); j < count;
+       j += wstride) {
+    int64_t i, slot;
+    if (j < ns) {
+      i = j;
+      slot = t0 + j;
+    } else {
+      i = iw + (j - ns);
+      const int64_t q = base + (j - ns);  // < 2 wr
+      slot = u.sink + (q >= wr ? q - wr : q);
+    }
+    const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * D) + lane * PER;
+    const int64_t rows[2] = {krow0 + slot, vrow0 + slot};
     const __nv_bfloat16* in[2] = {p.k, p.v};
+    uint32_t raw[2][PER / 2];
+#pragma unroll
+    for (int kv = 0; kv < 2; ++kv) {  // both loads in flight before any arithmetic
+      if constexpr (PER == 8) {
+        const uint4 v = *reinterpret_cast<const uint4*>(in[kv] + src);
+        raw[kv][0] = v.x; raw[kv][1] = v.y; raw[kv][2] = v.z; raw[kv][3] = v.w;
+      } else {
+        const uint2 v = *reinterpret_cast<const uint2*>(in[kv] + src);
+        raw[kv][0] = v.x; raw[kv][1] = v.y;
+      }
+    }
 #pragma unroll
     for (int kv = 0; kv < 2; ++kv) {
       float x[PER];
-      uint32_t raw[PER / 2];
-      if constexpr (PER == 8) {
-        const uint4 v = *reinterpret_cast<const uint4*>(in[kv] + src);
-        raw[0] = v.x; raw[1] = v.y; raw[2] = v.z; raw[3] = v.w;
-      } else {
-        const uint2 v = *reinterpret_cast<const uint2*>(in[kv] + src);
-        raw[0] = v.x; raw[1] = v.y;
-      }
 #pragma unroll
-      for (int j = 0; j < PER; ++j)
-        x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
+      for (int e = 0; e < PER; ++e)
+        x[e] = __uint_as_float((e & 1 ? raw[kv][e / 2] >> 16 : raw[kv][e / 2] & 0xffffu) << 16);
       uint32_t w[PER / 4];
       const float sc = e4m3_quantize_row_warp<PER>(x, w);
       uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + rows[kv] * D + lane * PER;
@@ -110,10 +125,14 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
 
 // Prefill staging for the 8-bit format, one warp per row, everything in fp16 for
 // an fp16 tensor-core pass. Ring rows: the held slots of (unit, batch row), below
-// min(t0, cap), dequantized (code x scale), and zeros for the next 128 slots, which
-// a key tile may read past them. Chunk K/V rows: quantized as append_fp8_kernel
-// stores them (same helper), then dequantized. q rows: converted. fp16 keeps 11
-// significant bits; magnitudes past its range saturate to +-65504.
+// min(t0, cap), and zeros for the next 128 slots, which a key tile may read past
+// them. Chunk K/V rows: quantized as append_fp8_kernel stores them (same helper).
+// K rows are staged as their code values (exact in fp16); their row scales stay
+// in fp32 (the arena's for ring rows, k_scale for chunk rows) and the prefill
+// kernel multiplies each logit by its key's scale, so no rounding of the scaled
+// key enters the logits. V rows are staged dequantized (code x scale, rounded to
+// fp16: 2^-11 relative on the values). q rows: converted. Magnitudes past the fp16
+// range saturate to +-65504.
 __device__ __forceinline__ void e4m3_words_to_f16(const uint32_t* words, int nwords, float sc,
                                                   uint32_t* out) {
   for (int i = 0; i < nwords; ++i) {
@@ -183,7 +202,7 @@ __global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) 
       } else {
         words[0] = *reinterpret_cast<const uint32_t*>(c);
       }
-      e4m3_words_to_f16(words, PER / 4, p.arena_scales[src], out);
+      e4m3_words_to_f16(words, PER / 4, kv ? p.arena_scales[src] : 1.f, out);
     }
     store_row16<PER>(p.ring + dst * D + lane * PER, out);
   }
@@ -198,8 +217,13 @@ __global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) 
       uint32_t w[PER / 4];
       const float sc = e4m3_quantize_row_warp<PER>(x, w);
       uint32_t out[PER / 2];
-      e4m3_words_to_f16(w, PER / 4, sc, out);
+      e4m3_words_to_f16(w, PER / 4, kv ? sc : 1.f, out);
       store_row16<PER>((kv ? p.v16 : p.k16) + off, out);
+      if (kv == 0 && lane == 0) {  // e = (b * n + i) * n_units + h
+        const int64_t h = e % p.n_units, bi = e / p.n_units;
+        const int64_t b = bi / p.n, i = bi - b * p.n;
+        p.k_scale[(b * p.n_units + h) * p.ks_ld + i] = sc;
+      }
     }
   }
   // q rows: index over (batch row, token, query head)
@@ -234,23 +258,24 @@ cudaError_t launch_fp8_stage(const Fp8StageParams& p, int head_dim, cudaStream_t
 }
 
 cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s) {
+  // blocks are laid out over (landing-row slice, KV head, batch row); grid x is sized for
+  // the head that keeps the most of the n new tokens (min(n, cap)); blocks past a head's
+  // own landing count exit at once
+  int64_t max_count = 0;
+  for (int h = 0; h < p.n_units; ++h) max_count = std::max(max_count, std::min(p.n, p.u[h].cap));
+  if (max_count == 0 || p.batch == 0) return cudaSuccess;
   if (fp8) {
-    const int64_t rows = (int64_t)p.batch * p.n * p.n_units;
-    if (rows == 0) return cudaSuccess;
-    int64_t blocks = (rows + 7) / 8;  // 8 warps per block, one row each
-    const int64_t cap_blocks = 152 * 16;
-    if (blocks > cap_blocks) blocks = cap_blocks;
+    int64_t blocks = (max_count + 31) / 32;  // 8 warps per block, up to 4 rows each
+    if (blocks > 65535) blocks = 65535;
+    const dim3 grid((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch);
     switch (p.d) {
-      case 128: return launch_pdl(append_fp8_kernel<128>, dim3((unsigned)blocks), dim3(256), 0, s, p);
-      case 256: return launch_pdl(append_fp8_kernel<256>, dim3((unsigned)blocks), dim3(256), 0, s, p);
+      case 128: return launch_pdl(append_fp8_kernel<128>, grid, dim3(256), 0, s, p);
+      case 256: return launch_pdl(append_fp8_kernel<256>, grid, dim3(256), 0, s, p);
       default: return cudaErrorInvalidValue;
     }
   }
-  const int64_t total = (int64_t)p.batch * p.n * p.n_units * (p.d / 8);
-  if (total == 0) return cudaSuccess;
-  // up to 4 vectors per thread for a head that keeps all n tokens; blocks of heads
-  // that keep fewer find no work and return
-  int64_t blocks = (p.n * (p.d / 8) + 1023) / 1024;
+  // up to 4 16-byte vectors per thread
+  int64_t blocks = (max_count * (p.d / 8) + 1023) / 1024;
   if (blocks > 65535) blocks = 65535;
   return launch_pdl(append_kernel, dim3((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch),
                     dim3(256), 0, s, p);

@@ -120,6 +120,9 @@ struct PrefillUnit {
   int64_t window;  // 0 = full
   int64_t stride;  // rows between batch rows
   int64_t sink;    // sink slots before the window region
+  // 8-bit cache: fp32 scale of ring slot j of batch row b of the call at
+  // ks_ring[ks_row0 + b * ks_stride + j] (the arena's K row scales)
+  int64_t ks_row0, ks_stride;
 };
 
 struct PrefillParams {
@@ -135,12 +138,19 @@ struct PrefillParams {
   const __nv_bfloat16* v_arena;
   float* out;               // [batch][n][n_q_heads][D]
   int* err;
+  // 8-bit cache (fp16 operand mode): the K tiles hold exact E4M3 code values and the
+  // logits of key j are multiplied by its row scale in fp32. Ring keys: the arena's
+  // scales (PrefillUnit::ks_row0); chunk keys: ks_chunk[(b * n_units + h) * ks_chunk_ld + i]
+  const float* ks_ring;
+  const float* ks_chunk;
+  int64_t ks_chunk_ld;
   PrefillUnit u[kMaxKvHeads];
 };
 
 // Staging of an 8-bit cache for prefill, everything in fp16 for an fp16 tensor-core
-// pass: the visible ring rows of one layer dequantized (code x scale), the chunk's
-// K/V rows quantized exactly as the append stores them and dequantized, and q.
+// pass: the visible ring rows of one layer (K as exact code values, V dequantized:
+// code x scale), the chunk's K/V rows quantized exactly as the append stores them
+// (K as code values with the row scales apart, V dequantized), and q.
 struct Fp8StageUnit {
   int64_t k_row0, v_row0, cap, stride, sink;  // arena rows
   int64_t sk_row0, sv_row0;                   // staging rows (batch row b at + b * cap)
@@ -157,6 +167,8 @@ struct Fp8StageParams {
   uint16_t* q16;                  // the same layouts, fp16
   uint16_t* k16;
   uint16_t* v16;
+  float* k_scale;                 // chunk K row scales [batch][n_units][ks_ld]
+  int64_t ks_ld;
   Fp8StageUnit u[kMaxKvHeads];
 };
 
@@ -397,6 +409,13 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
       : "=l"(d)
       : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)),
         "l"(*reinterpret_cast<uint64_t*>(&c)));
+  return *reinterpret_cast<float2*>(&d);
+}
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)));
   return *reinterpret_cast<float2*>(&d);
 }
 __device__ __forceinline__ float2 add2(float2 a, float2 b) {

@@ -90,3 +90,17 @@ def test_decode_bytes_8_bit_format():
     d = wl.head_dim
     # E4M3 codes (1 byte per channel) plus one fp32 scale per K and per V row
     assert fp8 * 4 * d == bf16 * 2 * (d + 4)
+
+
+def test_oracle_layer_steps_cover_every_unit():
+    """The oracle baseline times whole layer-steps: every (batch row, KV head) unit
+    of the layer, each over its whole retained window at position p."""
+    import oracle
+    wl = workloads.make("tiny")
+    orc = bench.OracleLayerSteps(wl, wl.max_ctx)
+    p = 300
+    sec, units, keys = orc.run_layer(0, p)
+    assert units == wl.batch * wl.n_kv_heads
+    assert keys == wl.batch * sum(p - oracle.window_lo(p, 0 if W >= wl.max_ctx else W) + 1
+                                  for W in wl.windows)
+    assert sec > 0
