@@ -64,9 +64,9 @@ typedef enum {
  *   HWKV_KV_BF16:     K and V rows in bf16 (b^K = b^V = 2 bytes).
  *   HWKV_KV_FP8_E4M3: K and V rows as 8-bit E4M3 codes (1 sign, 4 exponent bits
  *     with bias 7, 3 mantissa bits, largest finite 448) with one fp32 scale per
- *     stored row (one token of one KV head): s = amax / 448, code = nearest E4M3
- *     value of x / s (ties to even, saturating), value = code * s; a zero row
- *     stores s = 0. Effective precision (d + 4) / d bytes per element. Attention
+ *     stored row (one token of one KV head): s = the smallest power of two at or
+ *     above amax / 448 (amax / 448 in fp32), code = nearest E4M3 value of x / s
+ *     (ties to even, saturating), value = code * s; a zero row stores s = 0. Effective precision (d + 4) / d bytes per element. Attention
  *     reads the dequantised rows (the paper: when the format changes execution,
  *     every compared output uses it), in prefill the chunk's own keys included
  *     (they are read as the append stores them). head_dim 128 or 256.

@@ -31,8 +31,10 @@
  *                       this is a reading): E4M3 codes (1 sign bit, 4 exponent bits
  *                       with bias 7, 3 mantissa bits, no infinities, S.1111.111 =
  *                       NaN, largest finite 448) with one fp32 scale per stored row
- *                       (one token of one KV head): s = amax / 448, code = nearest
- *                       E4M3 value of x / s (ties to even, beyond 448 clamped to 448),
+ *                       (one token of one KV head): s = the smallest power of two
+ *                       >= amax / 448 (the shared power-of-two scale of the OCP
+ *                       microscaling formats, here per row), code = nearest E4M3
+ *                       value of x / s (ties to even, beyond 448 clamped to 448),
  *                       dequantised value decode(code) * s. Attention over such a
  *                       cache reads the dequantised rows (Sec. 3.1: when the format
  *                       changes execution, every compared output uses it).
@@ -451,8 +453,11 @@ uint8_t oracle_e4m3_encode(float x) {
 
 /*
  * One stored row in the 8-bit format: x[d] (bf16 bits) -> codes[d], *scale.
- * amax = max |x_i|; s = amax / 448 in float arithmetic; code_i = encode(x_i / s)
- * with x_i / s a float division; amax = 0 gives s = 0 and all-zero codes.
+ * amax = max |x_i|; r = amax / 448 in float arithmetic; s = the smallest power
+ * of two >= r (frexp: r = m 2^e with 1/2 <= m < 1, so s = r when m = 1/2, else
+ * 2^e); code_i = encode(x_i / s) with x_i / s a float division (exact, s being a
+ * power of two, up to the one rounding of a subnormal quotient); amax = 0 gives
+ * s = 0 and all-zero codes.
  */
 int oracle_quantize_row_e4m3(const uint16_t* x, int64_t d, uint8_t* codes, float* scale) {
   if (d <= 0) return 1;
@@ -466,7 +471,10 @@ int oracle_quantize_row_e4m3(const uint16_t* x, int64_t d, uint8_t* codes, float
     *scale = 0.0f;
     return 0;
   }
-  const volatile float s = amax / 448.0f;
+  const volatile float r = amax / 448.0f;
+  int e = 0;
+  const float m = frexpf(r, &e);
+  const volatile float s = m == 0.5f ? r : ldexpf(1.0f, e);
   for (int64_t i = 0; i < d; ++i) {
     const volatile float y = (float)bf16_to_double(x[i]) / s;
     codes[i] = oracle_e4m3_encode(y);

@@ -59,8 +59,9 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
 // The 8-bit format (E4M3 codes, one fp32 scale per stored row), laid out as the
 // bf16 kernel: block (x, h, b) takes the landing tokens of KV head h of batch row
 // b, one warp per token row (K and V), each lane D/32 consecutive channels.
-// amax = max |x|; s = amax / 448 (IEEE division); code = E4M3 of x / s (IEEE
-// division, round to nearest even, saturating); amax = 0 stores s = 0 and zeros.
+// amax = max |x|; s = the smallest power of two >= amax / 448; code = E4M3 of x / s
+// (an exact scaling; round to nearest even, saturating); amax = 0 stores s = 0 and
+// zeros (the shared row helper e4m3_quantize_row_warp).
 template <int D>
 __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   constexpr int PER = D / 32;
@@ -125,14 +126,13 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
 
 // Prefill staging for the 8-bit format, one warp per row, everything in fp16 for
 // an fp16 tensor-core pass. Ring rows: the held slots of (unit, batch row), below
-// min(t0, cap), and zeros for the next 128 slots, which a key tile may read past
-// them. Chunk K/V rows: quantized as append_fp8_kernel stores them (same helper).
-// K rows are staged as their code values (exact in fp16); their row scales stay
-// in fp32 (the arena's for ring rows, k_scale for chunk rows) and the prefill
-// kernel multiplies each logit by its key's scale, so no rounding of the scaled
-// key enters the logits. V rows are staged dequantized (code x scale, rounded to
-// fp16: 2^-11 relative on the values). q rows: converted. Magnitudes past the fp16
-// range saturate to +-65504.
+// min(t0, cap), dequantized (code x scale), and zeros for the next 128 slots, which
+// a key tile may read past them. Chunk K/V rows: quantized as append_fp8_kernel
+// stores them (same helper), then dequantized. q rows: converted. A code has at
+// most 4 significant bits and the row scale is a power of two, so code x scale is
+// exact in fp16 whenever it lies in fp16's range (at least 2^-24 for the smallest
+// code step, at most 65504); q in fp16 is exact for bf16 values of magnitude 2^-14
+// to 65504. Magnitudes past the fp16 range saturate to +-65504.
 __device__ __forceinline__ void e4m3_words_to_f16(const uint32_t* words, int nwords, float sc,
                                                   uint32_t* out) {
   for (int i = 0; i < nwords; ++i) {
@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) 
       } else {
         words[0] = *reinterpret_cast<const uint32_t*>(c);
       }
-      e4m3_words_to_f16(words, PER / 4, kv ? p.arena_scales[src] : 1.f, out);
+      e4m3_words_to_f16(words, PER / 4, p.arena_scales[src], out);
     }
     store_row16<PER>(p.ring + dst * D + lane * PER, out);
   }
@@ -217,13 +217,8 @@ __global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) 
       uint32_t w[PER / 4];
       const float sc = e4m3_quantize_row_warp<PER>(x, w);
       uint32_t out[PER / 2];
-      e4m3_words_to_f16(w, PER / 4, kv ? sc : 1.f, out);
+      e4m3_words_to_f16(w, PER / 4, sc, out);
       store_row16<PER>((kv ? p.v16 : p.k16) + off, out);
-      if (kv == 0 && lane == 0) {  // e = (b * n + i) * n_units + h
-        const int64_t h = e % p.n_units, bi = e / p.n_units;
-        const int64_t b = bi / p.n, i = bi - b * p.n;
-        p.k_scale[(b * p.n_units + h) * p.ks_ld + i] = sc;
-      }
     }
   }
   // q rows: index over (batch row, token, query head)

@@ -120,9 +120,6 @@ struct PrefillUnit {
   int64_t window;  // 0 = full
   int64_t stride;  // rows between batch rows
   int64_t sink;    // sink slots before the window region
-  // 8-bit cache: fp32 scale of ring slot j of batch row b of the call at
-  // ks_ring[ks_row0 + b * ks_stride + j] (the arena's K row scales)
-  int64_t ks_row0, ks_stride;
 };
 
 struct PrefillParams {
@@ -138,19 +135,12 @@ struct PrefillParams {
   const __nv_bfloat16* v_arena;
   float* out;               // [batch][n][n_q_heads][D]
   int* err;
-  // 8-bit cache (fp16 operand mode): the K tiles hold exact E4M3 code values and the
-  // logits of key j are multiplied by its row scale in fp32. Ring keys: the arena's
-  // scales (PrefillUnit::ks_row0); chunk keys: ks_chunk[(b * n_units + h) * ks_chunk_ld + i]
-  const float* ks_ring;
-  const float* ks_chunk;
-  int64_t ks_chunk_ld;
   PrefillUnit u[kMaxKvHeads];
 };
 
 // Staging of an 8-bit cache for prefill, everything in fp16 for an fp16 tensor-core
-// pass: the visible ring rows of one layer (K as exact code values, V dequantized:
-// code x scale), the chunk's K/V rows quantized exactly as the append stores them
-// (K as code values with the row scales apart, V dequantized), and q.
+// pass: the visible ring rows of one layer dequantized (code x scale), the chunk's
+// K/V rows quantized exactly as the append stores them and dequantized, and q.
 struct Fp8StageUnit {
   int64_t k_row0, v_row0, cap, stride, sink;  // arena rows
   int64_t sk_row0, sv_row0;                   // staging rows (batch row b at + b * cap)
@@ -167,8 +157,6 @@ struct Fp8StageParams {
   uint16_t* q16;                  // the same layouts, fp16
   uint16_t* k16;
   uint16_t* v16;
-  float* k_scale;                 // chunk K row scales [batch][n_units][ks_ld]
-  int64_t ks_ld;
   Fp8StageUnit u[kMaxKvHeads];
 };
 
@@ -354,10 +342,22 @@ __device__ __forceinline__ uint32_t f32x2_to_e4m3x2(float lo, float hi) {
   return d;
 }
 
+// Smallest power of two >= r, for a finite r > 0 below 2^127 (from the fp32 bits:
+// a normal r with a zero mantissa is a power of two already; otherwise the next
+// exponent; a subnormal r rounds its integer mantissa up to a power of two).
+__device__ __forceinline__ float pow2_ceil(float r) {
+  const uint32_t b = __float_as_uint(r);
+  const uint32_t ex = b >> 23, man = b & 0x7FFFFFu;
+  if (ex != 0) return man == 0 ? r : __uint_as_float((ex + 1u) << 23);
+  return __uint_as_float(man <= 1u ? man : 1u << (32 - __clz(man - 1u)));
+}
+
 // One row quantized to the 8-bit format by a warp, each lane holding PER of its
-// values: amax = max |x| over the row; s = amax / 448 (IEEE division); code =
-// E4M3 of x / s (IEEE division, round to nearest even, saturating); amax = 0 gives
-// s = 0 and zero codes. Returns s; w[i] packs the codes of x[4i .. 4i + 3].
+// values: amax = max |x| over the row; s = the smallest power of two >= amax / 448
+// (IEEE division); code = E4M3 of x / s (round to nearest even, saturating), where
+// x / s is an exact scaling, taken as x times the exact reciprocal of s (a division
+// when that reciprocal would not be a normal float); amax = 0 gives s = 0 and zero
+// codes. Returns s; w[i] packs the codes of x[4i .. 4i + 3].
 template <int PER>
 __device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], uint32_t (&w)[PER / 4]) {
   float amax = 0.f;
@@ -365,13 +365,21 @@ __device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], u
   for (int j = 0; j < PER; ++j) amax = fmaxf(amax, fabsf(x[j]));
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-  const float sc = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
+  const float sc = amax > 0.f ? pow2_ceil(__fdiv_rn(amax, 448.f)) : 0.f;
+  const uint32_t sex = __float_as_uint(sc) >> 23;  // exponent field of s
+  const bool mul = sex >= 1u && sex <= 253u;       // 1 / s is then a normal float
+  const float inv = __uint_as_float((254u - sex) << 23);
 #pragma unroll
   for (int j = 0; j < PER; j += 4) {
     uint32_t c01 = 0, c23 = 0;
     if (amax > 0.f) {
-      c01 = f32x2_to_e4m3x2(__fdiv_rn(x[j], sc), __fdiv_rn(x[j + 1], sc));
-      c23 = f32x2_to_e4m3x2(__fdiv_rn(x[j + 2], sc), __fdiv_rn(x[j + 3], sc));
+      if (mul) {
+        c01 = f32x2_to_e4m3x2(__fmul_rn(x[j], inv), __fmul_rn(x[j + 1], inv));
+        c23 = f32x2_to_e4m3x2(__fmul_rn(x[j + 2], inv), __fmul_rn(x[j + 3], inv));
+      } else {
+        c01 = f32x2_to_e4m3x2(__fdiv_rn(x[j], sc), __fdiv_rn(x[j + 1], sc));
+        c23 = f32x2_to_e4m3x2(__fdiv_rn(x[j + 2], sc), __fdiv_rn(x[j + 3], sc));
+      }
     }
     w[j / 4] = c01 | (c23 << 16);
   }
@@ -409,13 +417,6 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
       : "=l"(d)
       : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)),
         "l"(*reinterpret_cast<uint64_t*>(&c)));
-  return *reinterpret_cast<float2*>(&d);
-}
-__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
-  uint64_t d;
-  asm("mul.rn.f32x2 %0, %1, %2;"
-      : "=l"(d)
-      : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)));
   return *reinterpret_cast<float2*>(&d);
 }
 __device__ __forceinline__ float2 add2(float2 a, float2 b) {

@@ -74,16 +74,11 @@ struct TcCfg {
   // a softmax warp may run a key tile ahead of the PV issuer, so a per-tile barrier
   // could complete two phases before it is waited on), else one per query tile
   static constexpr int kPBars = PS ? QT * SBUF : QT;
-  // F16 (8-bit cache): the fp32 row scales of each K tile in a ring of their own, kept
-  // until the softmax has applied them (the K tile itself is free after its QK^T);
-  // a ring tile may start off a 16-byte boundary, so a slot holds BN + 4 scales
-  static constexpr int kKsc = F16 ? KST + 2 : 0;
-  static constexpr int kKsStride = BN + 4;
-  static constexpr int kScaleBytes = kKsc * kKsStride * 4;
-  static constexpr int kNumBars = 2 * KST + 2 * VST + 2 * QT * SBUF + 2 * kPBars + 2 * kKsc + 4;
-  static constexpr int kBarBytes = (8 * kNumBars + 4 + 127) / 128 * 128;  // + the TMEM address slot
+  static constexpr int kNumBars = 2 * KST + 2 * VST + 2 * QT * SBUF + 2 * kPBars + 4;
+  static constexpr int kBarBytes = 512;
+  static_assert(8 * kNumBars + 4 <= kBarBytes, "barriers and the TMEM address slot");
   // the dynamic shared memory window starts 1024-aligned (the kernel checks it)
-  static constexpr int kSmem = kQBytes + (KST + VST) * kTileBytes + kScaleBytes + kBarBytes;
+  static constexpr int kSmem = kQBytes + (KST + VST) * kTileBytes + kBarBytes;
   static_assert(kSmem * CTAS <= 232448 - 1024 * (CTAS - 1), "shared memory per SM");
   static constexpr int kTmemNeed = PS ? kColO + QT * D : kColO + QT * D + QT * BN / 2;
   // P of key chunk ch (64 keys = 32 columns) relative to col_p: chunk 0 first; with
@@ -247,8 +242,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
   uint8_t* sQ = smem;                                 // [QT] query tiles
   uint8_t* sK = smem + C::kQBytes;                   // [KST] K tiles
   uint8_t* sV = sK + KST * C::kTileBytes;            // [VST] V tiles
-  float* sKs = reinterpret_cast<float*>(sV + VST * C::kTileBytes);  // F16: [kKsc][kKsStride]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + VST * C::kTileBytes + C::kScaleBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + VST * C::kTileBytes);
   uint64_t* k_full = bars;                    // [KST] K tile landed
   uint64_t* k_empty = k_full + KST;           // [KST] QK^T of that tile done
   uint64_t* v_full = k_empty + KST;           // [VST] V tile landed
@@ -257,9 +251,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
   uint64_t* s_free = s_full + QT * SBUF;      // [QT][SBUF] S tile read by the softmax warps
   uint64_t* p_full = s_free + QT * SBUF;      // [kPBars] P written (and O rescaled)
   uint64_t* pv_done = p_full + C::kPBars;     // [kPBars] PV mma done
-  uint64_t* ks_full = pv_done + C::kPBars;    // F16: [kKsc] K-tile scales landed
-  uint64_t* ks_empty = ks_full + C::kKsc;     // F16: [kKsc] scales applied by every softmax warp
-  uint64_t* q_full = ks_empty + C::kKsc;
+  uint64_t* q_full = pv_done + C::kPBars;
   uint64_t* o_full = q_full + 1;
   uint64_t* drain = o_full + 1;               // [2] each issuer's mmas done
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
@@ -296,10 +288,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
       mbar_init(&p_full[i], 4);  // one arrival per warp of the tile's warpgroup
       mbar_init(&pv_done[i], 1);
     }
-    for (int i = 0; i < C::kKsc; ++i) {
-      mbar_init(&ks_full[i], 1);
-      mbar_init(&ks_empty[i], 4 * QT);  // every softmax warp of every query tile
-    }
     mbar_init(q_full, 1);
     mbar_init(o_full, 1);
     mbar_init(&drain[0], 1);
@@ -320,26 +308,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
   KeySeq<BN> seq;
   seq.init(u, t0, n_chunk, p0, p_last);
   bool aborted = false;
-  // F16: element index of the first scale of key tile (hist, j0) in its scale array;
-  // ring rows of a (unit, batch row) start on a 64-row boundary, chunk rows on a
-  // 128-entry one, so only a window-region tile of a sink head starts off 4 entries
-  auto ks_index = [&](int hist, int32_t j0) -> int64_t {
-    return hist ? u.ks_row0 + (int64_t)b * u.ks_stride + j0
-                : ((int64_t)b * p.n_units + h) * p.ks_chunk_ld + j0;
-  };
-  // F16: copy the scales of key tile `it` (BN + 4 from the 16-byte boundary at or below
-  // its first) into scale slot it mod kKsc, once every softmax warp is done with that slot
-  auto issue_scales = [&](uint32_t it, int hist, int32_t j0) {
-    if constexpr (C::kKsc > 0) {
-      const int ss = (int)(it % C::kKsc);
-      if (wait_or_abort(&ks_empty[ss], ((it / C::kKsc) & 1u) ^ 1u, p.err, aborted)) {
-        const int64_t e = ks_index(hist, j0);
-        const float* src = (hist ? p.ks_ring : p.ks_chunk) + (e & ~(int64_t)3);
-        mbar_arrive_expect_tx(&ks_full[ss], C::kKsStride * 4);
-        bulk_load(sKs + ss * C::kKsStride, src, C::kKsStride * 4, &ks_full[ss]);
-      }
-    }
-  };
 
   if (C::kSplitV && (warp == 0 || warp == C::kVWarp)) {
     // ------------------------------------------------- K and V producers (kSplitV)
@@ -375,7 +343,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
       int32_t j0;
       while (seq.next(hist, j0)) {
         const int s = it % nbuf;
-        if (is_k) issue_scales(it, hist, j0);
         if (wait_or_abort(&empty[s], ((it / nbuf) & 1u) ^ 1u, p.err, aborted)) {
           uint8_t* d = buf + s * C::kTileBytes;
           mbar_arrive_expect_tx(&full[s], C::kTileBytes);
@@ -422,13 +389,11 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
       KeySeq<BN> seq_v = seq;
       uint32_t it_k = 0, it_v = 0;
       auto issue = [&](KeySeq<BN>& sq, uint32_t& it, uint64_t* full, uint64_t* empty,
-                       uint8_t* buf, int64_t row0, const CUtensorMap* cmap, int nbuf,
-                       bool is_k) -> bool {
+                       uint8_t* buf, int64_t row0, const CUtensorMap* cmap, int nbuf) -> bool {
         int hist;
         int32_t j0;
         if (!sq.next(hist, j0)) return false;
         const int s = it % nbuf;
-        if (is_k) issue_scales(it, hist, j0);
         const uint32_t ph = (it / nbuf) & 1u;
         if (wait_or_abort(&empty[s], ph ^ 1u, p.err, aborted)) {
           uint8_t* d = buf + s * C::kTileBytes;
@@ -458,10 +423,10 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
       bool more_k = true;
       while (true) {
         while (more_k && lead <= kLead) {
-          more_k = issue(seq, it_k, k_full, k_empty, sK, krow0, &ck_map, KST, true);
+          more_k = issue(seq, it_k, k_full, k_empty, sK, krow0, &ck_map, KST);
           if (more_k) ++lead;
         }
-        if (!issue(seq_v, it_v, v_full, v_empty, sV, vrow0, &cv_map, VST, false)) break;
+        if (!issue(seq_v, it_v, v_full, v_empty, sV, vrow0, &cv_map, VST)) break;
         --lead;
       }
       // every issued copy has landed before shared memory can go away
@@ -602,14 +567,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
       const bool full_vis = !row_ok || (a0 <= 0 && b0 >= BN) || (a1 <= 0 && b1 >= BN);
       const bool warp_full = __all_sync(0xffffffffu, full_vis);  // warp-uniform fast path
       if (warp_wait_or_abort(&s_full[tq * SBUF + sb], (j / SBUF) & 1u, p.err, aborted)) tc_fence_after();
-      // F16: this key tile's scales (slot j mod kKsc, first at ks_off)
-      const float* ks_tile = sKs;
-      int ks_off = 0;
-      if constexpr (C::kKsc > 0) {
-        warp_wait_or_abort(&ks_full[j % C::kKsc], (j / C::kKsc) & 1u, p.err, aborted);
-        ks_off = (int)(ks_index(hist, j0) & 3);
-        ks_tile = sKs + (j % C::kKsc) * C::kKsStride + ks_off;
-      }
       // The S row in chunks of 64 columns: pass 1 takes the row max, pass 2 the
       // weights, the row sum and P. With one chunk the registers carry over; with
       // more the chunk is read from TMEM again (P over S overwrites only columns
@@ -620,26 +577,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
         tmem_ld32(t_lane + colS + sb * BN + ch * 64, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
         tmem_ld32(t_lane + colS + sb * BN + ch * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
         tmem_ld_wait();
-        if constexpr (C::kKsc > 0) {  // logit of key e = (q . code_e) x scale_e, in fp32
-          const float* ks = ks_tile + ch * 64;
-          if (ks_off == 0) {
-#pragma unroll
-            for (int e = 0; e < 64; e += 4) {
-              const float4 k4 = *reinterpret_cast<const float4*>(ks + e);
-              const float2 a = mul2(make_float2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])),
-                                    make_float2(k4.x, k4.y));
-              const float2 c2 = mul2(make_float2(__uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3])),
-                                     make_float2(k4.z, k4.w));
-              sv[e] = __float_as_uint(a.x);
-              sv[e + 1] = __float_as_uint(a.y);
-              sv[e + 2] = __float_as_uint(c2.x);
-              sv[e + 3] = __float_as_uint(c2.y);
-            }
-          } else {
-#pragma unroll
-            for (int e = 0; e < 64; ++e) sv[e] = __float_as_uint(__uint_as_float(sv[e]) * ks[e]);
-          }
-        }
         if (!warp_full) {  // masked logits -> -inf (weight 0)
 #pragma unroll
           for (int e = 0; e < 64; ++e) {
@@ -731,10 +668,6 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
         tmem_st32(t_lane + C::col_p(tq, j) + C::p_chunk_col(ch), *reinterpret_cast<const uint32_t(*)[32]>(&sv[0]));
       }
       tmem_st_wait();
-      if constexpr (C::kKsc > 0) {  // every read of this tile's scales is done
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&ks_empty[j % C::kKsc]);
-      }
       float s4[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
       const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
       l += sum;

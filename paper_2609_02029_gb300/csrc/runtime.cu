@@ -435,8 +435,6 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
     // a window that reaches past every position the kernel can see is the full history
     p.u[h] = PrefillUnit{u.k_row0, u.v_row0, u.cap, u.window >= ((int64_t)1 << 30) ? 0 : u.window,
                          u.stride, u.sink};
-    p.u[h].ks_row0 = u.k_row0 + (int64_t)row0 * u.stride;  // 8-bit: the arena's K row scales
-    p.u[h].ks_stride = u.stride;
   }
   // tensor maps of this call's q and chunk K/V: 3-D views {d, heads, batch * n}
   auto encode = get_encode();
@@ -498,11 +496,7 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
     const size_t ring_bytes = align_up((size_t)rows * d * 2, 1024);
     const size_t kv_bytes = align_up((size_t)n_rows * n * H * d * 2, 1024);
     const size_t q_bytes = align_up((size_t)n_rows * n * c->pol.n_q_heads * d * 2, 1024);
-    // chunk K row scales [row][KV head][n rounded up to 128], zero past n (a key tile
-    // reads whole 128-entry runs, plus 4 entries)
-    const int64_t ks_ld = (n + 127) / 128 * 128;
-    const size_t ks_bytes = align_up((size_t)n_rows * H * ks_ld * 4 + 64, 1024);
-    const size_t total = ring_bytes + 2 * kv_bytes + q_bytes + ks_bytes;
+    const size_t total = ring_bytes + 2 * kv_bytes + q_bytes;
     uint8_t* buf = nullptr;
     e = cudaMallocAsync(reinterpret_cast<void**>(&buf), total, s);
     if (e != cudaSuccess) return fail(HWKV_ENOMEM, "8-bit prefill staging (%zu bytes): %s", total, cudaGetErrorString(e));
@@ -510,10 +504,7 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
     sp.k16 = reinterpret_cast<uint16_t*>(buf + ring_bytes);
     sp.v16 = reinterpret_cast<uint16_t*>(buf + ring_bytes + kv_bytes);
     sp.q16 = reinterpret_cast<uint16_t*>(buf + ring_bytes + 2 * kv_bytes);
-    sp.k_scale = reinterpret_cast<float*>(buf + ring_bytes + 2 * kv_bytes + q_bytes);
-    sp.ks_ld = ks_ld;
-    e = cudaMemsetAsync(sp.k_scale, 0, ks_bytes, s);
-    if (e == cudaSuccess) e = launch_fp8_stage(sp, d, s);
+    e = launch_fp8_stage(sp, d, s);
     CUtensorMap ring_map, q16_map;
     CUresult r = CUDA_SUCCESS;
     if (e == cudaSuccess) {
@@ -544,9 +535,6 @@ hwkv_status hwkv_prefill_rows(hwkv_cache* c, int32_t layer, int32_t row0, int32_
         p.u[h].stride = sp.u[h].cap;
       }
       p.row0 = 0;
-      p.ks_ring = c->scales();
-      p.ks_chunk = sp.k_scale;
-      p.ks_chunk_ld = ks_ld;
       e = launch_prefill_tc(p, d, q16_map, ck_map, cv_map, ring_map, s, true);
     }
     const cudaError_t ef = cudaFreeAsync(buf, s);

@@ -2,7 +2,8 @@
 cache format; an 8-bit format changes execution, so attention reads the
 dequantised rows). The encoding is E4M3 (1 sign, 4 exponent bits with bias 7,
 3 mantissa bits, no infinities, S.1111.111 = NaN, largest finite 448) with one
-fp32 scale per stored row. Every pin follows from that definition, not from the
+fp32 scale per stored row, the smallest power of two at or above amax / 448 (the
+shared power-of-two scale of the OCP microscaling formats, taken per row). Every pin follows from that definition, not from the
 oracle's own code: values fixed by the format, round trips, ties to even at every
 midpoint, saturation, the rounding error bound, and a lossless case that must
 reproduce the bf16 attention oracle exactly."""
@@ -79,10 +80,14 @@ def test_row_quantization_bound_and_scale():
             xs = (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
             codes, s = oracle.quantize_row_e4m3(bits)
             amax = np.float32(np.abs(xs).max())
-            assert s == np.float32(amax / np.float32(448.0))
+            r = float(np.float32(amax / np.float32(448.0)))  # amax / 448 in float arithmetic
+            assert float(s) == 2.0 ** math.ceil(math.log2(r))  # smallest power of two >= r
+            assert math.frexp(float(s))[0] == 0.5 and r <= float(s) < 2 * r
             deq = np.array([oracle.e4m3_decode(c) for c in codes]) * float(s)
             i = int(np.argmax(np.abs(xs)))
-            assert codes[i] & 0x7F == 0x7E  # the largest element maps to +-448
+            assert 0x76 <= codes[i] & 0x7F <= 0x7E  # |x| / s in [224, 448]: the top binade
+            if scale >= 1.0:  # a 4-bit code times a power of two: exact in fp16 here
+                assert np.array_equal(deq.astype(np.float16).astype(np.float64), deq)
             # half a step: 2^-4 relative for normal codes, 2^-10 s for subnormal ones
             bound = np.maximum(np.abs(xs) * 2.0 ** -4, 2.0 ** -10 * float(s)) * (1 + 2.0 ** -18)
             assert np.all(np.abs(deq - xs) <= bound)
