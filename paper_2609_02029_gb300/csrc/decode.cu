@@ -81,27 +81,28 @@ __device__ __forceinline__ int dev_unit_len(const DecodeParams& p, int u, int32_
   return (int)(n < p.u[h].cap ? n : p.u[h].cap);
 }
 
-__device__ __forceinline__ long long warp_incl_scan(long long v, int lane) {
+__device__ __forceinline__ int warp_incl_scan(int v, int lane) {
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
-    const long long x = __shfl_up_sync(0xffffffffu, v, off);
+    const int x = __shfl_up_sync(0xffffffffu, v, off);
     if (lane >= off) v += x;
   }
   return v;
 }
 
-// called by whole warps; every lane returns the same plan
-__device__ __forceinline__ long long stages_of(long long n) {
-  return (n + kStageTokens - 1) / kStageTokens;
-}
+__device__ __forceinline__ int stages_of(int n) { return (n + kStageTokens - 1) / kStageTokens; }
 
+// Called by whole warps; every lane returns the same plan. Every count fits in 32
+// bits: a layer's keys are at most the arena's ring rows (below 2^30, which
+// hwkv_alloc checks), so its stages and the cost line stay below 2^26, and
+// c Lt / G is split as c (Lt / G) + c (Lt mod G) / G to stay in range.
 __device__ DevPlan make_device_plan(const DecodeParams& p, bool write_table) {
   const int lane = threadIdx.x & 31;
   const int U = p.batch * p.n_units;
   const int R = (U + 31) / 32;
-  const long long F = p.seg_cost;  // stages
+  const int F = p.seg_cost;  // stages
   int nreg[kPlanRegs];
-  long long Lt = 0, N = 0;
+  int Lt = 0, N = 0;
 #pragma unroll
   for (int r = 0; r < kPlanRegs; ++r) {
     const int u = r * 32 + lane;
@@ -133,15 +134,16 @@ __device__ DevPlan make_device_plan(const DecodeParams& p, bool write_table) {
     N += __shfl_xor_sync(0xffffffffu, N, off);
   }
 
-  const long long G = min((long long)gridDim.x, max(Lt, 1LL));
-  const bool mine = (long long)blockIdx.x < G && Lt > 0;
-  const long long A0 = mine ? (long long)blockIdx.x * Lt / G : 0;
-  const long long A1 = mine ? ((long long)blockIdx.x + 1) * Lt / G : 0;
+  const int G = min((int)gridDim.x, max(Lt, 1));
+  const int c = (int)blockIdx.x;
+  const bool mine = c < G && Lt > 0;
+  const int qL = Lt / G, rL = Lt - qL * G;
+  const int A0 = mine ? c * qL + (c * rL) / G : 0;                    // floor(c Lt / G)
+  const int A1 = mine ? (c + 1) * qL + ((c + 1) * rL) / G : 0;        // floor((c + 1) Lt / G)
   // line point -> key: the ring whose stretch [L_u, L_u + F + q_u) holds the point
-  long long a = -1, b = mine && A1 >= Lt ? N : -1;  // A1 = Lt: up to the last key
-  long long sa = 0;
-  int ua = 0;
-  long long carry_w = 0, carry_n = 0;
+  int a = -1, b = mine && A1 >= Lt ? N : -1;  // A1 = Lt: up to the last key
+  int sa = 0, ua = 0;
+  int carry_w = 0, carry_n = 0;
   for (int r = 0; r < R && ((mine && (a < 0 || b == -1)) || write_table); ++r) {
     int n = 0;
 #pragma unroll
@@ -152,9 +154,9 @@ __device__ DevPlan make_device_plan(const DecodeParams& p, bool write_table) {
       int32_t L;
       n = dev_unit_len(p, u, L);
     }
-    const long long w = n > 0 ? stages_of(n) + F : 0;
-    const long long iw = warp_incl_scan(w, lane), in = warp_incl_scan(n, lane);
-    const long long Lu = carry_w + iw - w, su = carry_n + in - n;
+    const int w = n > 0 ? stages_of(n) + F : 0;
+    const int iw = warp_incl_scan(w, lane), in = warp_incl_scan(n, lane);
+    const int Lu = carry_w + iw - w, su = carry_n + in - n;
     if (write_table && u < U) {
       p.plan[4 + 2 * u] = Lu;
       p.plan[5 + 2 * u] = n;
@@ -163,9 +165,9 @@ __device__ DevPlan make_device_plan(const DecodeParams& p, bool write_table) {
       const unsigned hit = __ballot_sync(0xffffffffu, w > 0 && Lu <= A0 && A0 < Lu + w);
       if (hit) {
         const int src = __ffs(hit) - 1;
-        const long long lu = __shfl_sync(0xffffffffu, Lu, src);
-        const long long s0 = __shfl_sync(0xffffffffu, su, src);
-        a = s0 + max(0LL, A0 - lu - F) * kStageTokens;
+        const int lu = __shfl_sync(0xffffffffu, Lu, src);
+        const int s0 = __shfl_sync(0xffffffffu, su, src);
+        a = s0 + max(0, A0 - lu - F) * kStageTokens;
         sa = s0;
         ua = r * 32 + src;
       }
@@ -174,9 +176,9 @@ __device__ DevPlan make_device_plan(const DecodeParams& p, bool write_table) {
       const unsigned hit = __ballot_sync(0xffffffffu, w > 0 && Lu <= A1 && A1 < Lu + w);
       if (hit) {
         const int src = __ffs(hit) - 1;
-        const long long lu = __shfl_sync(0xffffffffu, Lu, src);
-        const long long s1 = __shfl_sync(0xffffffffu, su, src);
-        b = s1 + max(0LL, A1 - lu - F) * kStageTokens;
+        const int lu = __shfl_sync(0xffffffffu, Lu, src);
+        const int s1 = __shfl_sync(0xffffffffu, su, src);
+        b = s1 + max(0, A1 - lu - F) * kStageTokens;
       }
     }
     carry_w += __shfl_sync(0xffffffffu, iw, 31);
@@ -685,18 +687,23 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
 
 // Log-sum-exp merge of the segment partials of one (batch row, query head):
 // o = sum_j 2^{(m_j - M) c} o_j / sum_j 2^{(m_j - M) c} l_j, M = max_j m_j.
-// One CTA of 8 warps per (batch row, query head): warp w sums partials w, w+8, ...
-// over all channels (each lane D/32 consecutive channels, vector loads); the
-// eight partial sums are added in shared memory in warp order (deterministic).
+// One CTA of 8 warps per (batch row, query head). Warp w merges partials w, w + 8,
+// w + 16, ... in that order with a running maximum (each lane D/32 consecutive
+// channels), loading a batch of partials (32 floats per lane) before using any of
+// them, so a ring
+// split over many CTAs costs a few rounds of L2 latency rather than one per
+// partial; the eight warps' results are then merged in warp order (deterministic).
 // Rings read whole by one CTA were written by the split kernel.
 constexpr int kCombineWarps = 8;
 
 template <int D>
 __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(const DecodeParams p) {
   constexpr int PER = D / 32;  // channels per lane
+  // partials loaded together; the registers stay low enough for a combine CTA to
+  // sit beside a split CTA on one SM (it launches early and waits there)
+  constexpr int kCombineBatch = 32 / PER;
   __shared__ float s_num[kCombineWarps][D];
-  __shared__ float s_den[kCombineWarps];
-  __shared__ float s_max[kCombineWarps];
+  __shared__ float2 s_ml[kCombineWarps];
   grid_dep_wait();  // partials come from the split kernel launched before
   const int bq = blockIdx.x;
   const int b = bq / p.n_q_heads;
@@ -729,44 +736,66 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
   const float c = p.scale_log2;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  float mx = -INFINITY;
-  for (int j = threadIdx.x; j < n_t; j += blockDim.x)
-    mx = fmaxf(mx, p.part_ml[slot(j) * kMaxGroup + n].x);
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  if (lane == 0) s_max[w] = mx;
-  __syncthreads();
-  float M = s_max[0];
-#pragma unroll
-  for (int k = 1; k < kCombineWarps; ++k) M = fmaxf(M, s_max[k]);
-
+  float m = -INFINITY, den = 0.f;
   float acc[PER];
 #pragma unroll
   for (int e = 0; e < PER; ++e) acc[e] = 0.f;
-  float den = 0.f;
-  for (int j = w; j < n_t; j += kCombineWarps) {
-    const float2 ml = p.part_ml[slot(j) * kMaxGroup + n];
-    const float wgt = ml.x == -INFINITY ? 0.f : ex2((ml.x - M) * c);
-    den += wgt * ml.y;
-    const float* src = p.part_o + (slot(j) * kMaxGroup + n) * D + lane * PER;
+  for (int j0 = w; j0 < n_t; j0 += kCombineBatch * kCombineWarps) {
+    float2 ml[kCombineBatch];
+    float v[kCombineBatch][PER];
 #pragma unroll
-    for (int e = 0; e < PER; e += 2) {
-      const float2 v = *reinterpret_cast<const float2*>(src + e);
-      acc[e] += wgt * v.x;
-      acc[e + 1] += wgt * v.y;
+    for (int k = 0; k < kCombineBatch; ++k) {
+      const int j = j0 + k * kCombineWarps;
+      if (j < n_t) {
+        const int64_t sl = slot(j);
+        ml[k] = p.part_ml[sl * kMaxGroup + n];
+        const float* src = p.part_o + (sl * kMaxGroup + n) * D + lane * PER;
+#pragma unroll
+        for (int e = 0; e < PER; e += 2) {
+          const float2 x = *reinterpret_cast<const float2*>(src + e);
+          v[k][e] = x.x;
+          v[k][e + 1] = x.y;
+        }
+      } else {
+        ml[k] = make_float2(-INFINITY, 0.f);
+#pragma unroll
+        for (int e = 0; e < PER; ++e) v[k][e] = 0.f;
+      }
     }
+    float mn = m;
+#pragma unroll
+    for (int k = 0; k < kCombineBatch; ++k) mn = fmaxf(mn, ml[k].x);
+    if (mn == -INFINITY) continue;  // nothing but empty partials so far
+    const float a = m == -INFINITY ? 0.f : ex2((m - mn) * c);
+    den *= a;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) acc[e] *= a;
+#pragma unroll
+    for (int k = 0; k < kCombineBatch; ++k) {
+      const float wk = ml[k].x == -INFINITY ? 0.f : ex2((ml[k].x - mn) * c);
+      den += wk * ml[k].y;
+#pragma unroll
+      for (int e = 0; e < PER; ++e) acc[e] += wk * v[k][e];
+    }
+    m = mn;
   }
 #pragma unroll
   for (int e = 0; e < PER; ++e) s_num[w][lane * PER + e] = acc[e];
-  if (lane == 0) s_den[w] = den;
+  if (lane == 0) s_ml[w] = make_float2(m, den);
   __syncthreads();
-  float dsum = 0.f;
+  float M = -INFINITY;
 #pragma unroll
-  for (int k = 0; k < kCombineWarps; ++k) dsum += s_den[k];
+  for (int k = 0; k < kCombineWarps; ++k) M = fmaxf(M, s_ml[k].x);
+  float wk[kCombineWarps], dsum = 0.f;
+#pragma unroll
+  for (int k = 0; k < kCombineWarps; ++k) {
+    wk[k] = s_ml[k].x == -INFINITY ? 0.f : ex2((s_ml[k].x - M) * c);
+    dsum += wk[k] * s_ml[k].y;
+  }
   for (int i = threadIdx.x; i < D; i += blockDim.x) {
     float num = 0.f;
 #pragma unroll
-    for (int k = 0; k < kCombineWarps; ++k) num += s_num[k][i];
+    for (int k = 0; k < kCombineWarps; ++k) num += wk[k] * s_num[k][i];
     p.out[((int64_t)b * p.n_q_heads + qh) * D + i] = num / dsum;
   }
 }
