@@ -524,7 +524,7 @@ def run_prefill(args, local, fp8=False, workload="prefill64k"):
 
 
 # ------------------------------------------------------------ GPU append
-def run_append(local, n=8192, reps=10, warm=3, fp8=False):
+def run_append(local, n=8192, reps=10, warm=3, fp8=False, batch=0):
     """hwkv_append of 8,192-token chunks into layer 0 of layers16_112k (batch 16,
     4 KV heads, d 256, rings of {full, 32768, 8192, 2048, 512} drawn per head):
     each call reads the chunk's K and V (537 MB, more than L2) and writes the last
@@ -544,7 +544,7 @@ def run_append(local, n=8192, reps=10, warm=3, fp8=False):
     stream = torch.cuda.current_stream(dev)
     s = stream.cuda_stream
     g = hwkv_gen.desc(wl.seed, wl.per_head_scale)
-    B, Hkv, d = wl.batch, wl.n_kv_heads, wl.head_dim
+    B, Hkv, d = (batch or wl.batch), wl.n_kv_heads, wl.head_dim
     windows = wl.windows[:Hkv]
     k = torch.empty((B, n, Hkv, d), dtype=torch.bfloat16, device=dev)
     v = torch.empty_like(k)
@@ -572,7 +572,8 @@ def run_append(local, n=8192, reps=10, warm=3, fp8=False):
     ms = float(np.median(times))
     del k, v, arena
     torch.cuda.empty_cache()
-    return {"workload": "layers16_112k layer 0, 8192-token chunks" + (", 8-bit cache" if fp8 else ""),
+    return {"workload": "layers16_112k layer 0, 8192-token chunks" + (", 8-bit cache" if fp8 else "")
+                        + (", batch %d" % B if batch else ""),
             "ms": ms,
             "bytes_per_call": per_call, "gbs": per_call / (ms * 1e-3) / 1e9}
 
@@ -826,7 +827,7 @@ def main():
         return
 
     if args.append_only:
-        a = run_append(local, fp8=args.kv == "fp8")
+        a = run_append(local, fp8=args.kv == "fp8", batch=args.batch)
         emit({"metric": "append GB/s", "value": a["gbs"], "unit": "GB/s", "n_gpus": 1,
               "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
               "config": {"workload": a["workload"]}, "ms": a["ms"],

@@ -16,6 +16,7 @@
 namespace hwkv {
 
 __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
+  grid_dep_launch();  // the next kernel may start its prologue (it waits for this one)
   grid_dep_wait();  // k/v may come from the kernel launched before; the previous
                     // decode of this ring must be done reading before slots are reused
   if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && p.lens != nullptr)
@@ -58,14 +59,15 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
 
 // The 8-bit format (E4M3 codes, one fp32 scale per stored row), laid out as the
 // bf16 kernel: block (x, h, b) takes the landing tokens of KV head h of batch row
-// b; a warp quantizes whole token rows (K and V), each lane D/32 consecutive
-// channels, four rows at a time.
+// b; a warp quantizes one token row (K and V) at a time, each lane D/32 consecutive
+// channels.
 // amax = max |x|; s = the smallest power of two >= amax / 448; code = E4M3 of x / s
 // (an exact scaling; round to nearest even, saturating); amax = 0 stores s = 0 and
 // zeros (the shared row helper e4m3_quantize_row_warp).
 template <int D>
 __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   constexpr int PER = D / 32;
+  grid_dep_launch();
   grid_dep_wait();
   if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && p.lens != nullptr)
     for (int b = threadIdx.x; b < p.batch; b += blockDim.x)
@@ -81,59 +83,46 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   const int64_t base = iw < n ? (t0 + iw - u.sink) % wr : 0;  // window slot of token iw
   const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;
   const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.stride;
-  // warp-slot w takes the landing rows w, w + W, w + 2W, w + 3W (W = warps in the
-  // grid's x slice), loading all four before quantizing any, then moves on by 4W
-  constexpr int kRows = 4;
   const int64_t wstride = (int64_t)gridDim.x * (blockDim.x / 32);
-  for (int64_t j0 = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); j0 < count;
-       j0 += kRows * wstride) {
-    uint32_t raw[kRows][2][PER / 2];
-    int64_t slot[kRows];
+  for (int64_t j = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); j < count;
+       j += wstride) {
+    int64_t i, slot;
+    if (j < ns) {
+      i = j;
+      slot = t0 + j;
+    } else {
+      i = iw + (j - ns);
+      const int64_t q = base + (j - ns);  // < 2 wr
+      slot = u.sink + (q >= wr ? q - wr : q);
+    }
+    const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * D) + lane * PER;
+    const int64_t rows[2] = {krow0 + slot, vrow0 + slot};
+    const __nv_bfloat16* in[2] = {p.k, p.v};
+    uint32_t raw[2][PER / 2];
 #pragma unroll
-    for (int r = 0; r < kRows; ++r) {
-      const int64_t j = j0 + r * wstride;
-      if (j >= count) break;
-      int64_t i;
-      if (j < ns) {
-        i = j;
-        slot[r] = t0 + j;
+    for (int kv = 0; kv < 2; ++kv) {  // both loads in flight before any arithmetic
+      if constexpr (PER == 8) {
+        const uint4 v = *reinterpret_cast<const uint4*>(in[kv] + src);
+        raw[kv][0] = v.x; raw[kv][1] = v.y; raw[kv][2] = v.z; raw[kv][3] = v.w;
       } else {
-        i = iw + (j - ns);
-        const int64_t q = base + (j - ns);  // < 2 wr
-        slot[r] = u.sink + (q >= wr ? q - wr : q);
-      }
-      const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * D) + lane * PER;
-#pragma unroll
-      for (int kv = 0; kv < 2; ++kv) {
-        const __nv_bfloat16* in = (kv ? p.v : p.k) + src;
-        if constexpr (PER == 8) {
-          const uint4 v = *reinterpret_cast<const uint4*>(in);
-          raw[r][kv][0] = v.x; raw[r][kv][1] = v.y; raw[r][kv][2] = v.z; raw[r][kv][3] = v.w;
-        } else {
-          const uint2 v = *reinterpret_cast<const uint2*>(in);
-          raw[r][kv][0] = v.x; raw[r][kv][1] = v.y;
-        }
+        const uint2 v = *reinterpret_cast<const uint2*>(in[kv] + src);
+        raw[kv][0] = v.x; raw[kv][1] = v.y;
       }
     }
 #pragma unroll
-    for (int r = 0; r < kRows; ++r) {
-      if (j0 + r * wstride >= count) break;
+    for (int kv = 0; kv < 2; ++kv) {
+      float x[PER];
 #pragma unroll
-      for (int kv = 0; kv < 2; ++kv) {
-        float x[PER];
-#pragma unroll
-        for (int e = 0; e < PER; ++e)
-          x[e] = __uint_as_float((e & 1 ? raw[r][kv][e / 2] >> 16 : raw[r][kv][e / 2] & 0xffffu) << 16);
-        uint32_t w[PER / 4];
-        const float sc = e4m3_quantize_row_warp<PER>(x, w);
-        const int64_t row = (kv ? vrow0 : krow0) + slot[r];
-        uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + row * D + lane * PER;
-        if constexpr (PER == 8)
-          *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
-        else
-          *reinterpret_cast<uint32_t*>(dst) = w[0];
-        if (lane == 0) p.scales[row] = sc;
-      }
+      for (int e = 0; e < PER; ++e)
+        x[e] = __uint_as_float((e & 1 ? raw[kv][e / 2] >> 16 : raw[kv][e / 2] & 0xffffu) << 16);
+      uint32_t w[PER / 4];
+      const float sc = e4m3_quantize_row_warp<PER>(x, w);
+      uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + rows[kv] * D + lane * PER;
+      if constexpr (PER == 8)
+        *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
+      else
+        *reinterpret_cast<uint32_t*>(dst) = w[0];
+      if (lane == 0) p.scales[rows[kv]] = sc;
     }
   }
 }
@@ -274,7 +263,7 @@ cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s) {
   for (int h = 0; h < p.n_units; ++h) max_count = std::max(max_count, std::min(p.n, p.u[h].cap));
   if (max_count == 0 || p.batch == 0) return cudaSuccess;
   if (fp8) {
-    int64_t blocks = (max_count + 31) / 32;  // 8 warps per block, 4 rows each
+    int64_t blocks = (max_count + 31) / 32;  // 8 warps per block, up to 4 rows each
     if (blocks > 65535) blocks = 65535;
     const dim3 grid((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch);
     switch (p.d) {

@@ -324,6 +324,17 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
     }
     fence_barrier_init();
   }
+  // Before waiting for the kernel launched before (this launch may start while it
+  // runs): the unit table and the tensor maps do not depend on it, so bring them
+  // into the constant cache now
+  if (p.tiles == nullptr && lane < p.n_units) {
+    const DecodeUnit& du = p.u[lane];
+    asm volatile("" ::"l"(du.k_row0), "l"(du.v_row0), "l"(du.cap), "l"(du.stride), "l"(du.sink));
+  }
+  if (warp == kDecodeWarps && lane == 0) {
+    prefetch_tensormap(&k_map);
+    prefetch_tensormap(&v_map);
+  }
   __syncthreads();
   grid_dep_wait();    // the ring append, q and the lengths come from kernels launched before
   grid_dep_launch();  // the combine kernel may start launching
