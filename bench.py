@@ -37,10 +37,11 @@ from hwkv_gen import workloads  # noqa: E402
 NOMINAL_HBM_GBS = 8000.0
 L2_BYTES = 129 * 1024 * 1024
 # DRAM bytes (read + write) per algorithmic byte of the decode split kernel, from an ncu
-# capture (--set full) of the 1-layer, batch-2 case of layers16_112k;
-# traffic is reads of every resident K/V row plus tile partials, so it scales with the
-# algorithmic bytes of a launch. Set to None whenever that kernel changes.
-DECODE_TRAFFIC_PER_BYTE = (244.301312e6 + 3.917312e6) / 244066304.0
+# capture (--set full) of the 1-layer, batch-2 case of layers16_112k
+# (profiles/decode_split_small_full.md); traffic is reads of every resident K/V row plus
+# segment partials, so it scales with the algorithmic bytes of a launch. Set to None
+# whenever that kernel changes.
+DECODE_TRAFFIC_PER_BYTE = (244.291584e6 + 4.332032e6) / 244064256.0
 # tensor-pipe activity of the prefill kernel (ncu sm__pipe_tensor_cycles_active, pct of peak
 # sustained active) from the one-launch --set full capture summarised in the named profile;
 # set to None whenever that kernel changes.

@@ -352,12 +352,19 @@ __device__ __forceinline__ float pow2_ceil(float r) {
   return __uint_as_float(man <= 1u ? man : 1u << (32 - __clz(man - 1u)));
 }
 
-// One row quantized to the 8-bit format by a warp, each lane holding PER of its
-// values: amax = max |x| over the row; s = the smallest power of two >= amax / 448
-// (IEEE division); code = E4M3 of x / s (round to nearest even, saturating), where
-// x / s is an exact scaling, taken as x times the exact reciprocal of s (a division
-// when that reciprocal would not be a normal float); amax = 0 gives s = 0 and zero
-// codes. Returns s; w[i] packs the codes of x[4i .. 4i + 3].
+// One row of bf16 values quantized to the 8-bit format by a warp, each lane holding
+// PER of them: amax = max |x| over the row; s = the smallest power of two >= amax / 448
+// (amax / 448 rounded to fp32, as the format defines it); code = E4M3 of x / s (round
+// to nearest even, saturating), where x / s is an exact scaling, taken as x times the
+// exact reciprocal of s (a division when that reciprocal would not be a normal float);
+// amax = 0 gives s = 0 and zero codes. Returns s; w[i] packs the codes of x[4i .. 4i+3].
+//
+// s comes from amax's bits without a division. Write amax = (1 + f) 2^e with f in
+// [0, 1) and 448 = 1.75 2^8. If 1 + f <= 1.75, amax / 448 lies in (2^(e-9), 2^(e-8)]
+// and s = 2^(e-8); otherwise it lies in (2^(e-8), 2^(e-7)) and s = 2^(e-7). Rounding
+// amax / 448 to fp32 cannot cross those powers of two: amax is a bf16 value (7 fraction
+// bits), so unless 1 + f = 1.75 exactly (quotient exactly 2^(e-8)) the quotient is at
+// least a factor 1.0044 away from each of them, far beyond fp32 rounding.
 template <int PER>
 __device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], uint32_t (&w)[PER / 4]) {
   float amax = 0.f;
@@ -365,7 +372,12 @@ __device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], u
   for (int j = 0; j < PER; ++j) amax = fmaxf(amax, fabsf(x[j]));
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-  const float sc = amax > 0.f ? pow2_ceil(__fdiv_rn(amax, 448.f)) : 0.f;
+  const uint32_t ab = __float_as_uint(amax), aex = ab >> 23;
+  float sc = 0.f;
+  if (aex > 8u)  // s = 2^(e-8) or 2^(e-7) is a normal float
+    sc = __uint_as_float(((ab & 0x7FFFFFu) <= 0x600000u ? aex - 8u : aex - 7u) << 23);
+  else if (amax > 0.f)
+    sc = pow2_ceil(__fdiv_rn(amax, 448.f));
   const uint32_t sex = __float_as_uint(sc) >> 23;  // exponent field of s
   const bool mul = sex >= 1u && sex <= 253u;       // 1 / s is then a normal float
   const float inv = __uint_as_float((254u - sex) << 23);
