@@ -58,22 +58,23 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
 }
 
 // The 8-bit format (E4M3 codes, one fp32 scale per stored row), laid out as the
-// bf16 kernel: block (x, h, b) takes the landing tokens of KV head h of batch row
-// b; a warp quantizes one token row (K and V) at a time, each lane D/32 consecutive
-// channels.
+// bf16 kernel: block (x, h, b) takes the landing tokens of KV head h of batch row b;
+// each half warp quantizes one token row (K and V), each lane D/16 consecutive
+// channels (a half-warp row needs one shuffle step less per value than a warp row
+// and spreads each row's index arithmetic over twice the values).
 // amax = max |x|; s = the smallest power of two >= amax / 448; code = E4M3 of x / s
 // (an exact scaling; round to nearest even, saturating); amax = 0 stores s = 0 and
 // zeros (the shared row helper e4m3_quantize_row_warp).
 template <int D>
 __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
-  constexpr int PER = D / 32;
+  constexpr int PER = D / 16;  // values per lane
   grid_dep_launch();
   grid_dep_wait();
   if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && p.lens != nullptr)
     for (int b = threadIdx.x; b < p.batch; b += blockDim.x)
       p.lens[p.row0 + b] = (int32_t)(p.t0[b] + p.n);
   const int h = blockIdx.y, b = blockIdx.z;
-  const int lane = threadIdx.x & 31;
+  const int hl = threadIdx.x & 15;  // lane within the half warp
   const AppendUnit& u = p.u[h];
   const int64_t n = p.n, t0 = p.t0[b];
   const int64_t wr = u.cap - u.sink;
@@ -83,9 +84,15 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   const int64_t base = iw < n ? (t0 + iw - u.sink) % wr : 0;  // window slot of token iw
   const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;
   const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.stride;
-  const int64_t wstride = (int64_t)gridDim.x * (blockDim.x / 32);
-  for (int64_t j = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); j < count;
-       j += wstride) {
+  // half warp g takes rows g, g + H, ... (H = the half warps of the grid's x slice); both
+  // halves of a warp make the same trips (a row past the end is read clamped and not
+  // stored) so the shuffles of the row maximum stay converged
+  const int64_t hstride = (int64_t)gridDim.x * (blockDim.x / 16);
+  const int half = (threadIdx.x >> 4) & 1;
+  for (int64_t jw = (int64_t)blockIdx.x * (blockDim.x / 16) + (threadIdx.x >> 4) - half; jw < count;
+       jw += hstride) {
+    const bool valid = jw + half < count;
+    const int64_t j = valid ? jw + half : count - 1;
     int64_t i, slot;
     if (j < ns) {
       i = j;
@@ -95,34 +102,31 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
       const int64_t q = base + (j - ns);  // < 2 wr
       slot = u.sink + (q >= wr ? q - wr : q);
     }
-    const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * D) + lane * PER;
-    const int64_t rows[2] = {krow0 + slot, vrow0 + slot};
-    const __nv_bfloat16* in[2] = {p.k, p.v};
-    uint32_t raw[2][PER / 2];
-#pragma unroll
-    for (int kv = 0; kv < 2; ++kv) {  // both loads in flight before any arithmetic
-      if constexpr (PER == 8) {
-        const uint4 v = *reinterpret_cast<const uint4*>(in[kv] + src);
-        raw[kv][0] = v.x; raw[kv][1] = v.y; raw[kv][2] = v.z; raw[kv][3] = v.w;
-      } else {
-        const uint2 v = *reinterpret_cast<const uint2*>(in[kv] + src);
-        raw[kv][0] = v.x; raw[kv][1] = v.y;
-      }
-    }
+    const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * D) + hl * PER;
 #pragma unroll
     for (int kv = 0; kv < 2; ++kv) {
+      const __nv_bfloat16* in = (kv ? p.v : p.k) + src;
+      uint32_t raw[PER / 2];
+#pragma unroll
+      for (int c = 0; c < PER / 8; ++c) {
+        const uint4 v4 = *reinterpret_cast<const uint4*>(in + c * 8);
+        raw[4 * c] = v4.x; raw[4 * c + 1] = v4.y; raw[4 * c + 2] = v4.z; raw[4 * c + 3] = v4.w;
+      }
       float x[PER];
 #pragma unroll
       for (int e = 0; e < PER; ++e)
-        x[e] = __uint_as_float((e & 1 ? raw[kv][e / 2] >> 16 : raw[kv][e / 2] & 0xffffu) << 16);
+        x[e] = __uint_as_float((e & 1 ? raw[e / 2] >> 16 : raw[e / 2] & 0xffffu) << 16);
       uint32_t w[PER / 4];
-      const float sc = e4m3_quantize_row_warp<PER>(x, w);
-      uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + rows[kv] * D + lane * PER;
-      if constexpr (PER == 8)
-        *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
-      else
-        *reinterpret_cast<uint32_t*>(dst) = w[0];
-      if (lane == 0) p.scales[rows[kv]] = sc;
+      const float sc = e4m3_quantize_row_warp<PER, 16>(x, w);
+      if (valid) {
+        const int64_t row = (kv ? vrow0 : krow0) + slot;
+        uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + row * D + hl * PER;
+        if constexpr (PER == 16)
+          *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+        else
+          *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
+        if (hl == 0) p.scales[row] = sc;
+      }
     }
   }
 }
@@ -263,7 +267,7 @@ cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s) {
   for (int h = 0; h < p.n_units; ++h) max_count = std::max(max_count, std::min(p.n, p.u[h].cap));
   if (max_count == 0 || p.batch == 0) return cudaSuccess;
   if (fp8) {
-    int64_t blocks = (max_count + 31) / 32;  // 8 warps per block, up to 4 rows each
+    int64_t blocks = (max_count + 63) / 64;  // 16 half warps per block, up to 4 rows each
     if (blocks > 65535) blocks = 65535;
     const dim3 grid((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch);
     switch (p.d) {

@@ -352,8 +352,8 @@ __device__ __forceinline__ float pow2_ceil(float r) {
   return __uint_as_float(man <= 1u ? man : 1u << (32 - __clz(man - 1u)));
 }
 
-// One row of bf16 values quantized to the 8-bit format by a warp, each lane holding
-// PER of them: amax = max |x| over the row; s = the smallest power of two >= amax / 448
+// One row of bf16 values quantized to the 8-bit format by LANES lanes (a warp, or
+// each half of one with LANES = 16), each lane holding PER of them: amax = max |x| over the row; s = the smallest power of two >= amax / 448
 // (amax / 448 rounded to fp32, as the format defines it); code = E4M3 of x / s (round
 // to nearest even, saturating), where x / s is an exact scaling, taken as x times the
 // exact reciprocal of s (a division when that reciprocal would not be a normal float);
@@ -365,13 +365,14 @@ __device__ __forceinline__ float pow2_ceil(float r) {
 // amax / 448 to fp32 cannot cross those powers of two: amax is a bf16 value (7 fraction
 // bits), so unless 1 + f = 1.75 exactly (quotient exactly 2^(e-8)) the quotient is at
 // least a factor 1.0044 away from each of them, far beyond fp32 rounding.
-template <int PER>
+template <int PER, int LANES = 32>
 __device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], uint32_t (&w)[PER / 4]) {
+  static_assert(LANES == 32 || LANES == 16, "a warp or half a warp per row");
   float amax = 0.f;
 #pragma unroll
   for (int j = 0; j < PER; ++j) amax = fmaxf(amax, fabsf(x[j]));
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+  for (int off = LANES / 2; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
   const uint32_t ab = __float_as_uint(amax), aex = ab >> 23;
   float sc = 0.f;
   if (aex > 8u)  // s = 2^(e-8) or 2^(e-7) is a normal float

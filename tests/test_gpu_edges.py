@@ -1,7 +1,8 @@
 """Parity at the edges of the supported sizes, through the C ABI against the oracle:
-the largest KV-head count (64) with the largest GQA group (8, so 512 query heads),
-the largest batch (256 rows) through prefill and the fused decode step, and empty
-calls (n = 0 appends and prefills change nothing)."""
+the largest KV-head count (64) and the largest GQA group (8), each with 256 query
+heads (the input generator keys at most 256 heads), the largest batch (256 rows)
+through prefill and the fused decode step, and empty calls (n = 0 appends and
+prefills change nothing)."""
 import numpy as np
 import pytest
 
@@ -12,20 +13,22 @@ from harness import Run, assert_close, check_ring_unit, oracle_unit_decode
 pytestmark = pytest.mark.gpu
 
 
-def test_64_kv_heads_group_8():
-    windows = [0 if h % 4 == 0 else (17 * h + 3) for h in range(64)]
-    r = Run(1, 1, 512, 64, 64, 420, windows, seed=41)
+@pytest.mark.parametrize("Hkv,G", [(64, 4), (32, 8)])
+def test_most_kv_heads_and_largest_group(Hkv, G):
+    windows = [0 if h % 4 == 0 else (17 * h + 3) for h in range(Hkv)]
+    Hq = Hkv * G
+    r = Run(1, 1, Hq, Hkv, 64, 420, windows, seed=41)
     try:
         out = r.prefill(0, 390).cpu().numpy()
         rows = [0, 1, 100, 257, 388, 389]
-        for qh in range(0, 512, 37):
+        for qh in range(0, Hq, 37):
             assert_close(out[0, rows, qh], r.oracle_rows(0, 0, qh, rows), "prefill q%d" % qh)
         for _ in range(3):
             got = r.decode_step_fused(0).cpu().numpy()
         p = hwkv.hwkv_seq_len(r.cache, 0) - 1
-        for h in range(64):
-            assert_close(got[0, h * 8:(h + 1) * 8], oracle_unit_decode(r, 0, 0, h, p), "decode h%d" % h)
-        for h in (0, 1, 63):
+        for h in range(Hkv):
+            assert_close(got[0, h * G:(h + 1) * G], oracle_unit_decode(r, 0, 0, h, p), "decode h%d" % h)
+        for h in (0, 1, Hkv - 1):
             check_ring_unit(r, 0, 0, h)
         r.check_residency()
         hwkv.hwkv_sync_check(r.cache)
