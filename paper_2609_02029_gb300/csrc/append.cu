@@ -89,45 +89,58 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   // stored) so the shuffles of the row maximum stay converged
   const int64_t hstride = (int64_t)gridDim.x * (blockDim.x / 16);
   const int half = (threadIdx.x >> 4) & 1;
+  constexpr int ROWS = 2;  // rows per half warp and trip, all their loads in flight at once
   for (int64_t jw = (int64_t)blockIdx.x * (blockDim.x / 16) + (threadIdx.x >> 4) - half; jw < count;
-       jw += hstride) {
-    const bool valid = jw + half < count;
-    const int64_t j = valid ? jw + half : count - 1;
-    int64_t i, slot;
-    if (j < ns) {
-      i = j;
-      slot = t0 + j;
-    } else {
-      i = iw + (j - ns);
-      const int64_t q = base + (j - ns);  // < 2 wr
-      slot = u.sink + (q >= wr ? q - wr : q);
-    }
-    const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * D) + hl * PER;
+       jw += ROWS * hstride) {
+    bool valid[ROWS];
+    int64_t slot[ROWS];
+    // K and V loads of every row before any arithmetic: the stores below go through
+    // the arena pointer, which the compiler cannot tell apart from p.k and p.v
+    uint32_t raw[ROWS][2][PER / 2];
 #pragma unroll
-    for (int kv = 0; kv < 2; ++kv) {
-      const __nv_bfloat16* in = (kv ? p.v : p.k) + src;
-      uint32_t raw[PER / 2];
-#pragma unroll
-      for (int c = 0; c < PER / 8; ++c) {
-        const uint4 v4 = *reinterpret_cast<const uint4*>(in + c * 8);
-        raw[4 * c] = v4.x; raw[4 * c + 1] = v4.y; raw[4 * c + 2] = v4.z; raw[4 * c + 3] = v4.w;
+    for (int r = 0; r < ROWS; ++r) {
+      const int64_t j0 = jw + r * hstride + half;
+      valid[r] = j0 < count;
+      const int64_t j = valid[r] ? j0 : count - 1;
+      int64_t i;
+      if (j < ns) {
+        i = j;
+        slot[r] = t0 + j;
+      } else {
+        i = iw + (j - ns);
+        const int64_t q = base + (j - ns);  // < 2 wr
+        slot[r] = u.sink + (q >= wr ? q - wr : q);
       }
-      float x[PER];
+      const int64_t src = ((((int64_t)b * n + i) * p.n_units + h) * D) + hl * PER;
 #pragma unroll
-      for (int e = 0; e < PER; ++e)
-        x[e] = __uint_as_float((e & 1 ? raw[e / 2] >> 16 : raw[e / 2] & 0xffffu) << 16);
-      uint32_t w[PER / 4];
-      const float sc = e4m3_quantize_row_warp<PER, 16>(x, w);
-      if (valid) {
-        const int64_t row = (kv ? vrow0 : krow0) + slot;
-        uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + row * D + hl * PER;
-        if constexpr (PER == 16)
-          *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
-        else
-          *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
-        if (hl == 0) p.scales[row] = sc;
-      }
+      for (int kv = 0; kv < 2; ++kv)
+#pragma unroll
+        for (int c = 0; c < PER / 8; ++c) {
+          const uint4 v4 = *reinterpret_cast<const uint4*>((kv ? p.v : p.k) + src + c * 8);
+          raw[r][kv][4 * c] = v4.x; raw[r][kv][4 * c + 1] = v4.y;
+          raw[r][kv][4 * c + 2] = v4.z; raw[r][kv][4 * c + 3] = v4.w;
+        }
     }
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r)
+#pragma unroll
+      for (int kv = 0; kv < 2; ++kv) {
+        float x[PER];
+#pragma unroll
+        for (int e = 0; e < PER; ++e)
+          x[e] = __uint_as_float((e & 1 ? raw[r][kv][e / 2] >> 16 : raw[r][kv][e / 2] & 0xffffu) << 16);
+        uint32_t w[PER / 4];
+        const float sc = e4m3_quantize_row_warp<PER, 16>(x, w);
+        if (valid[r]) {
+          const int64_t row = (kv ? vrow0 : krow0) + slot[r];
+          uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + row * D + hl * PER;
+          if constexpr (PER == 16)
+            *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+          else
+            *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
+          if (hl == 0) p.scales[row] = sc;
+        }
+      }
   }
 }
 
@@ -267,7 +280,10 @@ cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s) {
   for (int h = 0; h < p.n_units; ++h) max_count = std::max(max_count, std::min(p.n, p.u[h].cap));
   if (max_count == 0 || p.batch == 0) return cudaSuccess;
   if (fp8) {
-    int64_t blocks = (max_count + 63) / 64;  // 16 half warps per block, up to 4 rows each
+    // 16 half warps per block, up to kFp8RowsPerHalfWarp rows each (fewer, longer-lived
+    // blocks measured faster than one or two trips per half warp)
+    constexpr int64_t kFp8RowsPerHalfWarp = 8;
+    int64_t blocks = (max_count + 16 * kFp8RowsPerHalfWarp - 1) / (16 * kFp8RowsPerHalfWarp);
     if (blocks > 65535) blocks = 65535;
     const dim3 grid((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch);
     switch (p.d) {
