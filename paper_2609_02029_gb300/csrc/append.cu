@@ -125,12 +125,8 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
     for (int r = 0; r < ROWS; ++r)
 #pragma unroll
       for (int kv = 0; kv < 2; ++kv) {
-        float x[PER];
-#pragma unroll
-        for (int e = 0; e < PER; ++e)
-          x[e] = __uint_as_float((e & 1 ? raw[r][kv][e / 2] >> 16 : raw[r][kv][e / 2] & 0xffffu) << 16);
         uint32_t w[PER / 4];
-        const float sc = e4m3_quantize_row_warp<PER, 16>(x, w);
+        const float sc = e4m3_quantize_row_warp<PER, 16>(raw[r][kv], w);
         if (valid[r]) {
           const int64_t row = (kv ? vrow0 : krow0) + slot[r];
           uint8_t* dst = reinterpret_cast<uint8_t*>(p.k_arena) + row * D + hl * PER;
@@ -172,8 +168,7 @@ __device__ __forceinline__ void store_row16(uint16_t* dst, const uint32_t (&w)[P
     *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
 }
 template <int PER>
-__device__ __forceinline__ void load_row_bf16(const __nv_bfloat16* src, float (&x)[PER]) {
-  uint32_t raw[PER / 2];
+__device__ __forceinline__ void load_row_bf16(const __nv_bfloat16* src, uint32_t (&raw)[PER / 2]) {
   if constexpr (PER == 8) {
     const uint4 v = *reinterpret_cast<const uint4*>(src);
     raw[0] = v.x; raw[1] = v.y; raw[2] = v.z; raw[3] = v.w;
@@ -181,9 +176,6 @@ __device__ __forceinline__ void load_row_bf16(const __nv_bfloat16* src, float (&
     const uint2 v = *reinterpret_cast<const uint2*>(src);
     raw[0] = v.x; raw[1] = v.y;
   }
-#pragma unroll
-  for (int j = 0; j < PER; ++j)
-    x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
 }
 
 template <int D>
@@ -232,10 +224,10 @@ __global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) 
     const int64_t off = e * D + lane * PER;
 #pragma unroll
     for (int kv = 0; kv < 2; ++kv) {
-      float x[PER];
-      load_row_bf16<PER>((kv ? p.v : p.k) + off, x);
+      uint32_t raw[PER / 2];
+      load_row_bf16<PER>((kv ? p.v : p.k) + off, raw);
       uint32_t w[PER / 4];
-      const float sc = e4m3_quantize_row_warp<PER>(x, w);
+      const float sc = e4m3_quantize_row_warp<PER>(raw, w);
       uint32_t out[PER / 2];
       e4m3_words_to_f16(w, PER / 4, sc, out);
       store_row16<PER>((kv ? p.v16 : p.k16) + off, out);
@@ -245,11 +237,12 @@ __global__ void __launch_bounds__(256) fp8_stage_kernel(const Fp8StageParams p) 
   const int64_t q_items = (int64_t)p.batch * p.n * p.n_q_heads;
   for (int64_t e = warp0; e < q_items; e += warps) {
     const int64_t off = e * D + lane * PER;
-    float x[PER];
-    load_row_bf16<PER>(p.q + off, x);
+    uint32_t raw[PER / 2];
+    load_row_bf16<PER>(p.q + off, raw);
     uint32_t out[PER / 2];
 #pragma unroll
-    for (int i = 0; i < PER / 2; ++i) out[i] = pack_f16_sat(x[2 * i], x[2 * i + 1]);
+    for (int i = 0; i < PER / 2; ++i)
+      out[i] = pack_f16_sat(__uint_as_float(raw[i] << 16), __uint_as_float(raw[i] & 0xffff0000u));
     store_row16<PER>(p.q16 + off, out);
   }
 }

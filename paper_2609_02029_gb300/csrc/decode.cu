@@ -475,12 +475,8 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
               const uint2 v = *reinterpret_cast<const uint2*>(src);
               raw[0] = v.x; raw[1] = v.y;
             }
-            float x[PER];
-#pragma unroll
-            for (int j = 0; j < PER; ++j)
-              x[j] = __uint_as_float((j & 1 ? raw[j / 2] >> 16 : raw[j / 2] & 0xffffu) << 16);
             uint32_t cw[PER / 4];
-            const float sc = e4m3_quantize_row_warp<PER>(x, cw);
+            const float sc = e4m3_quantize_row_warp<PER>(raw, cw);
             const int64_t ring = (kv ? ti.v_row : ti.k_row) - ti.start + ti.s_new;
             uint8_t* g = reinterpret_cast<uint8_t*>(p.arena) + ring * D + lane * PER;
             const int c0 = lane * PER;  // first channel of this lane

@@ -352,12 +352,31 @@ __device__ __forceinline__ float pow2_ceil(float r) {
   return __uint_as_float(man <= 1u ? man : 1u << (32 - __clz(man - 1u)));
 }
 
+// packed fp32 pair product (sm_100+), each lane rounded to nearest even
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)));
+  return *reinterpret_cast<float2*>(&d);
+}
+
+// Larger magnitude of two bf16 pairs, lane by lane (exact; the sign bits carry the
+// xor of the operands' signs, which callers drop)
+__device__ __forceinline__ uint32_t bf16x2_absmax(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.xorsign.abs.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
 // One row of bf16 values quantized to the 8-bit format by LANES lanes (a warp, or
-// each half of one with LANES = 16), each lane holding PER of them: amax = max |x| over the row; s = the smallest power of two >= amax / 448
-// (amax / 448 rounded to fp32, as the format defines it); code = E4M3 of x / s (round
-// to nearest even, saturating), where x / s is an exact scaling, taken as x times the
-// exact reciprocal of s (a division when that reciprocal would not be a normal float);
-// amax = 0 gives s = 0 and zero codes. Returns s; w[i] packs the codes of x[4i .. 4i+3].
+// each half of one with LANES = 16), each lane holding PER of them as PER / 2 packed
+// pairs (element 2i in the low half of raw[i]): amax = max |x| over the row; s = the
+// smallest power of two >= amax / 448 (amax / 448 rounded to fp32, as the format
+// defines it); code = E4M3 of x / s (round to nearest even, saturating), where x / s is
+// an exact scaling, taken as x times the exact reciprocal of s (a division when that
+// reciprocal would not be a normal float); amax = 0 gives s = 0 and zero codes.
+// Returns s; w[i] packs the codes of elements 4i .. 4i+3.
 //
 // s comes from amax's bits without a division. Write amax = (1 + f) 2^e with f in
 // [0, 1) and 448 = 1.75 2^8. If 1 + f <= 1.75, amax / 448 lies in (2^(e-9), 2^(e-8)]
@@ -365,12 +384,21 @@ __device__ __forceinline__ float pow2_ceil(float r) {
 // amax / 448 to fp32 cannot cross those powers of two: amax is a bf16 value (7 fraction
 // bits), so unless 1 + f = 1.75 exactly (quotient exactly 2^(e-8)) the quotient is at
 // least a factor 1.0044 away from each of them, far beyond fp32 rounding.
+//
+// The maximum is taken on the packed pairs and the scaling on fp32 pairs: both are
+// exact, so the codes are those of the elementwise definition.
 template <int PER, int LANES = 32>
-__device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], uint32_t (&w)[PER / 4]) {
+__device__ __forceinline__ float e4m3_quantize_row_warp(const uint32_t (&raw)[PER / 2], uint32_t (&w)[PER / 4]) {
   static_assert(LANES == 32 || LANES == 16, "a warp or half a warp per row");
-  float amax = 0.f;
+  static_assert(PER % 4 == 0, "codes are packed four to a word");
+  uint32_t mw[PER / 2];
 #pragma unroll
-  for (int j = 0; j < PER; ++j) amax = fmaxf(amax, fabsf(x[j]));
+  for (int i = 0; i < PER / 2; ++i) mw[i] = raw[i];
+#pragma unroll
+  for (int span = PER / 4; span > 0; span >>= 1)  // pairwise tree over the words
+#pragma unroll
+    for (int i = 0; i < span; ++i) mw[i] = bf16x2_absmax(mw[i], mw[i + span]);
+  float amax = fmaxf(fabsf(__uint_as_float(mw[0] << 16)), fabsf(__uint_as_float(mw[0] & 0xffff0000u)));
 #pragma unroll
   for (int off = LANES / 2; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
   const uint32_t ab = __float_as_uint(amax), aex = ab >> 23;
@@ -382,19 +410,24 @@ __device__ __forceinline__ float e4m3_quantize_row_warp(const float (&x)[PER], u
   const uint32_t sex = __float_as_uint(sc) >> 23;  // exponent field of s
   const bool mul = sex >= 1u && sex <= 253u;       // 1 / s is then a normal float
   const float inv = __uint_as_float((254u - sex) << 23);
+  const float2 inv2 = make_float2(inv, inv);
 #pragma unroll
-  for (int j = 0; j < PER; j += 4) {
+  for (int i = 0; i < PER / 2; i += 2) {
+    float2 x01 = make_float2(__uint_as_float(raw[i] << 16), __uint_as_float(raw[i] & 0xffff0000u));
+    float2 x23 = make_float2(__uint_as_float(raw[i + 1] << 16), __uint_as_float(raw[i + 1] & 0xffff0000u));
     uint32_t c01 = 0, c23 = 0;
     if (amax > 0.f) {
       if (mul) {
-        c01 = f32x2_to_e4m3x2(__fmul_rn(x[j], inv), __fmul_rn(x[j + 1], inv));
-        c23 = f32x2_to_e4m3x2(__fmul_rn(x[j + 2], inv), __fmul_rn(x[j + 3], inv));
+        x01 = mul2(x01, inv2);
+        x23 = mul2(x23, inv2);
       } else {
-        c01 = f32x2_to_e4m3x2(__fdiv_rn(x[j], sc), __fdiv_rn(x[j + 1], sc));
-        c23 = f32x2_to_e4m3x2(__fdiv_rn(x[j + 2], sc), __fdiv_rn(x[j + 3], sc));
+        x01 = make_float2(__fdiv_rn(x01.x, sc), __fdiv_rn(x01.y, sc));
+        x23 = make_float2(__fdiv_rn(x23.x, sc), __fdiv_rn(x23.y, sc));
       }
+      c01 = f32x2_to_e4m3x2(x01.x, x01.y);
+      c23 = f32x2_to_e4m3x2(x23.x, x23.y);
     }
-    w[j / 4] = c01 | (c23 << 16);
+    w[i / 2] = c01 | (c23 << 16);
   }
   return sc;
 }

@@ -14,7 +14,7 @@ class Run:
     """One cache plus the device buffers needed to drive it."""
 
     def __init__(self, n_layers, batch, n_q_heads, n_kv_heads, head_dim, max_ctx, windows,
-                 seed=0, per_head_scale=False):
+                 seed=0, per_head_scale=False, kv_format=hwkv.HWKV_KV_BF16):
         import torch
         self.torch = torch
         self.L, self.B, self.Hq, self.Hkv, self.d = n_layers, batch, n_q_heads, n_kv_heads, head_dim
@@ -24,7 +24,7 @@ class Run:
         self.g = hwkv_gen.desc(seed, per_head_scale)
         self.scale = 1.0 / np.sqrt(head_dim)
         self.pol = hwkv.make_policy(n_layers, n_kv_heads, n_q_heads, head_dim, batch, max_ctx,
-                                    windows)
+                                    windows, kv_format=kv_format)
         self.nbytes = hwkv.hwkv_required_bytes(self.pol)
         self.arena = torch.empty(self.nbytes, dtype=torch.uint8, device="cuda")
         self.stream = torch.cuda.current_stream()
