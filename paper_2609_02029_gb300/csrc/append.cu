@@ -19,13 +19,16 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
   grid_dep_launch();  // the next kernel may start its prologue (it waits for this one)
   grid_dep_wait();  // k/v may come from the kernel launched before; the previous
                     // decode of this ring must be done reading before slots are reused
-  if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && p.lens != nullptr)
+  if (blockIdx.x == 0 && blockIdx.z == 0 && p.lens != nullptr)
     for (int b = threadIdx.x; b < p.batch; b += blockDim.x)  // nothing in this grid reads them
       p.lens[p.row0 + b] = (int32_t)(p.t0[b] + p.n);
-  // block (x, h, b): KV head h of batch row b. Of the n new tokens only these land:
-  // the ns that are sink positions (< sink, slot = position) and, of the rest, the
-  // last wr (window-region slots), whose slots follow each other from one base mod wr
-  const int h = blockIdx.y, b = blockIdx.z;
+  // block (x, b): a block of KV head h's range of batch row b. Of the n new tokens only
+  // these land: the ns that are sink positions (< sink, slot = position) and, of the
+  // rest, the last wr (window-region slots), whose slots follow each other from one base
+  // mod wr
+  const int h = append_block_head(p, (int32_t)blockIdx.x), b = blockIdx.z;
+  const int64_t xb = (int64_t)blockIdx.x - p.blk0[h];    // block within the head's range
+  const int64_t nb = (int64_t)p.blk0[h + 1] - p.blk0[h];  // blocks of the head's range
   const AppendUnit& u = p.u[h];
   const int64_t n = p.n, t0 = p.t0[b];
   const int64_t wr = u.cap - u.sink;
@@ -37,8 +40,7 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
   const int64_t vmask = (1 << vpr_log2) - 1;
   const int64_t krow0 = u.k_row0 + (int64_t)(p.row0 + b) * u.stride;
   const int64_t vrow0 = u.v_row0 + (int64_t)(p.row0 + b) * u.stride;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < (count << vpr_log2);
-       e += (int64_t)gridDim.x * blockDim.x) {
+  for (int64_t e = xb * blockDim.x + threadIdx.x; e < (count << vpr_log2); e += nb * blockDim.x) {
     const int64_t j = e >> vpr_log2, vec = e & vmask;
     int64_t i, slot;
     if (j < ns) {
@@ -70,10 +72,12 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   constexpr int PER = D / 16;  // values per lane
   grid_dep_launch();
   grid_dep_wait();
-  if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && p.lens != nullptr)
+  if (blockIdx.x == 0 && blockIdx.z == 0 && p.lens != nullptr)
     for (int b = threadIdx.x; b < p.batch; b += blockDim.x)
       p.lens[p.row0 + b] = (int32_t)(p.t0[b] + p.n);
-  const int h = blockIdx.y, b = blockIdx.z;
+  const int h = append_block_head(p, (int32_t)blockIdx.x), b = blockIdx.z;
+  const int64_t xb = (int64_t)blockIdx.x - p.blk0[h];    // block within the head's range
+  const int64_t nb = (int64_t)p.blk0[h + 1] - p.blk0[h];  // blocks of the head's range
   const int hl = threadIdx.x & 15;  // lane within the half warp
   const AppendUnit& u = p.u[h];
   const int64_t n = p.n, t0 = p.t0[b];
@@ -87,10 +91,10 @@ __global__ void __launch_bounds__(256) append_fp8_kernel(const AppendParams p) {
   // half warp g takes rows g, g + H, ... (H = the half warps of the grid's x slice); both
   // halves of a warp make the same trips (a row past the end is read clamped and not
   // stored) so the shuffles of the row maximum stay converged
-  const int64_t hstride = (int64_t)gridDim.x * (blockDim.x / 16);
+  const int64_t hstride = nb * (blockDim.x / 16);
   const int half = (threadIdx.x >> 4) & 1;
   constexpr int ROWS = 2;  // rows per half warp and trip, all their loads in flight at once
-  for (int64_t jw = (int64_t)blockIdx.x * (blockDim.x / 16) + (threadIdx.x >> 4) - half; jw < count;
+  for (int64_t jw = xb * (blockDim.x / 16) + (threadIdx.x >> 4) - half; jw < count;
        jw += ROWS * hstride) {
     bool valid[ROWS];
     int64_t slot[ROWS];
@@ -265,31 +269,33 @@ cudaError_t launch_fp8_stage(const Fp8StageParams& p, int head_dim, cudaStream_t
   return cudaGetLastError();
 }
 
-cudaError_t launch_append(const AppendParams& p, bool fp8, cudaStream_t s) {
-  // blocks are laid out over (landing-row slice, KV head, batch row); grid x is sized for
-  // the head that keeps the most of the n new tokens (min(n, cap)); blocks past a head's
-  // own landing count exit at once
-  int64_t max_count = 0;
-  for (int h = 0; h < p.n_units; ++h) max_count = std::max(max_count, std::min(p.n, p.u[h].cap));
-  if (max_count == 0 || p.batch == 0) return cudaSuccess;
+cudaError_t launch_append(const AppendParams& p0, bool fp8, cudaStream_t s) {
+  // grid x of a batch row is laid out head by head, each head sized for the most rows it
+  // can take (min(n, cap)); a block past its row's own landing count exits at once.
+  // bf16: up to 4 16-byte vectors per thread. 8-bit: 16 half warps per block, up to
+  // kFp8RowsPerHalfWarp rows each (fewer, longer-lived blocks measured faster than one or
+  // two trips per half warp).
+  constexpr int64_t kFp8RowsPerHalfWarp = 8;
+  AppendParams p = p0;
+  int64_t total = 0;
+  for (int h = 0; h < p.n_units; ++h) {
+    const int64_t rows = std::min(p.n, p.u[h].cap);
+    p.blk0[h] = (int32_t)total;
+    total += fp8 ? (rows + 16 * kFp8RowsPerHalfWarp - 1) / (16 * kFp8RowsPerHalfWarp)
+                 : (rows * (p.d / 8) + 1023) / 1024;
+    if (total >= (int64_t)INT32_MAX) return cudaErrorInvalidValue;
+  }
+  p.blk0[p.n_units] = (int32_t)total;
+  if (total == 0 || p.batch == 0) return cudaSuccess;
+  const dim3 grid((unsigned)total, 1, (unsigned)p.batch);
   if (fp8) {
-    // 16 half warps per block, up to kFp8RowsPerHalfWarp rows each (fewer, longer-lived
-    // blocks measured faster than one or two trips per half warp)
-    constexpr int64_t kFp8RowsPerHalfWarp = 8;
-    int64_t blocks = (max_count + 16 * kFp8RowsPerHalfWarp - 1) / (16 * kFp8RowsPerHalfWarp);
-    if (blocks > 65535) blocks = 65535;
-    const dim3 grid((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch);
     switch (p.d) {
       case 128: return launch_pdl(append_fp8_kernel<128>, grid, dim3(256), 0, s, p);
       case 256: return launch_pdl(append_fp8_kernel<256>, grid, dim3(256), 0, s, p);
       default: return cudaErrorInvalidValue;
     }
   }
-  // up to 4 16-byte vectors per thread
-  int64_t blocks = (max_count * (p.d / 8) + 1023) / 1024;
-  if (blocks > 65535) blocks = 65535;
-  return launch_pdl(append_kernel, dim3((unsigned)blocks, (unsigned)p.n_units, (unsigned)p.batch),
-                    dim3(256), 0, s, p);
+  return launch_pdl(append_kernel, grid, dim3(256), 0, s, p);
 }
 
 }  // namespace hwkv

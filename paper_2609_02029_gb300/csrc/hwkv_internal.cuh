@@ -112,7 +112,20 @@ struct AppendParams {
   __nv_bfloat16* v_arena;
   float* scales;           // 8-bit format: scale of row r at scales[r]
   AppendUnit u[kMaxKvHeads];
+  // grid x of one batch row: KV head h owns blocks [blk0[h], blk0[h + 1]), sized for its
+  // own landing rows (at most min(n, cap))
+  int32_t blk0[kMaxKvHeads + 1];
 };
+
+// KV head whose block range [blk0[h], blk0[h + 1]) holds block x (x < blk0[n_units])
+__device__ __forceinline__ int append_block_head(const AppendParams& p, int32_t x) {
+  int lo = 0, hi = p.n_units - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.blk0[mid] <= x) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
 
 // ------------------------------------------------------------------ prefill
 struct PrefillUnit {
