@@ -694,25 +694,29 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
 
 // Log-sum-exp merge of the segment partials of one (batch row, query head):
 // o = sum_j 2^{(m_j - M) c} o_j / sum_j 2^{(m_j - M) c} l_j, M = max_j m_j.
-// One CTA of 8 warps per (batch row, query head). Warp w merges partials w, w + 8,
-// w + 16, ... in that order with a running maximum (each lane D/32 consecutive
-// channels), loading a batch of partials (32 floats per lane) before using any of
-// them, so a ring
-// split over many CTAs costs a few rounds of L2 latency rather than one per
-// partial; the eight warps' results are then merged in warp order (deterministic).
-// Rings read whole by one CTA were written by the split kernel.
+// CH CTAs of 8 warps per (batch row, query head), each over D / CH consecutive
+// channels (CH > 1 for small steps, with few (batch row, query head) pairs: the merge
+// is spread over more SMs and each warp takes more partials per round). Warp w merges partials w, w + 8, w + 16, ... in that order with a running
+// maximum (each lane D / (32 CH) consecutive channels), loading a batch of partials
+// (32 floats per lane) before using any of them, so a ring split over many CTAs costs
+// a few rounds of L2 latency rather than one per partial; the eight warps' results
+// are then merged in warp order (deterministic). Rings read whole by one CTA were
+// written by the split kernel.
 constexpr int kCombineWarps = 8;
 
-template <int D>
+template <int D, int CH>
 __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(const DecodeParams p) {
-  constexpr int PER = D / 32;  // channels per lane
+  constexpr int DC = D / CH;    // channels of this CTA
+  constexpr int PER = DC / 32;  // channels per lane
+  static_assert(PER >= 2 && PER % 2 == 0, "channel pairs per lane");
   // partials loaded together; the registers stay low enough for a combine CTA to
   // sit beside a split CTA on one SM (it launches early and waits there)
   constexpr int kCombineBatch = 32 / PER;
-  __shared__ float s_num[kCombineWarps][D];
+  __shared__ float s_num[kCombineWarps][DC];
   __shared__ float2 s_ml[kCombineWarps];
   grid_dep_wait();  // partials come from the split kernel launched before
-  const int bq = blockIdx.x;
+  const int bq = blockIdx.x / CH;
+  const int c0 = (blockIdx.x - bq * CH) * DC;  // first channel of this CTA
   const int b = bq / p.n_q_heads;
   const int qh = bq - b * p.n_q_heads;
   const int h = qh / p.group;
@@ -726,11 +730,11 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
   const long long Lu = p.plan[4 + 2 * u], nu = p.plan[5 + 2 * u];
   // every ring of an active row holds >= 1 key; the split kernel has finished
   // reading the lengths, so the row can advance now
-  if (p.lens_inc && qh == 0 && threadIdx.x == 0 && p.plan[5 + 2 * (b * p.n_units)] > 0)
+  if (p.lens_inc && qh == 0 && c0 == 0 && threadIdx.x == 0 && p.plan[5 + 2 * (b * p.n_units)] > 0)
     p.lens[b] += 1;
   if (nu == 0) {  // idle row (or a row at max_ctx): zero output
-    for (int i = threadIdx.x; i < D; i += blockDim.x)
-      p.out[((int64_t)b * p.n_q_heads + qh) * D + i] = 0.f;
+    for (int i = threadIdx.x; i < DC; i += blockDim.x)
+      p.out[((int64_t)b * p.n_q_heads + qh) * D + c0 + i] = 0.f;
     return;
   }
   const long long qu = (nu + kStageTokens - 1) / kStageTokens;
@@ -756,7 +760,7 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
       if (j < n_t) {
         const int64_t sl = slot(j);
         ml[k] = p.part_ml[sl * kMaxGroup + n];
-        const float* src = p.part_o + (sl * kMaxGroup + n) * D + lane * PER;
+        const float* src = p.part_o + (sl * kMaxGroup + n) * D + c0 + lane * PER;
 #pragma unroll
         for (int e = 0; e < PER; e += 2) {
           const float2 x = *reinterpret_cast<const float2*>(src + e);
@@ -799,11 +803,11 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
     wk[k] = s_ml[k].x == -INFINITY ? 0.f : ex2((s_ml[k].x - M) * c);
     dsum += wk[k] * s_ml[k].y;
   }
-  for (int i = threadIdx.x; i < D; i += blockDim.x) {
+  for (int i = threadIdx.x; i < DC; i += blockDim.x) {
     float num = 0.f;
 #pragma unroll
     for (int k = 0; k < kCombineWarps; ++k) num += wk[k] * s_num[k][i];
-    p.out[((int64_t)b * p.n_q_heads + qh) * D + i] = num / dsum;
+    p.out[((int64_t)b * p.n_q_heads + qh) * D + c0 + i] = num / dsum;
   }
 }
 
@@ -1016,12 +1020,21 @@ cudaError_t launch_wait_probe(int* err, uint64_t limit_ns, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s) {
-  const dim3 grid(p.batch * p.n_q_heads), block(kCombineWarps * 32);
+cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, int num_sms, cudaStream_t s) {
+  // at most a quarter as many (batch row, query head) pairs as SMs (a small step, whose
+  // rings are cut into many segments): each pair's channels over D / 64 CTAs; with more
+  // pairs the extra CTAs measured slower (batch 4 at 161K: 1-2% per step)
+  const int pairs = p.batch * p.n_q_heads;
+  const bool split = 4 * pairs <= num_sms && head_dim >= 128;
+  const dim3 block(kCombineWarps * 32);
   switch (head_dim) {
-    case 64: return launch_pdl(decode_combine_kernel<64>, grid, block, 0, s, p);
-    case 128: return launch_pdl(decode_combine_kernel<128>, grid, block, 0, s, p);
-    case 256: return launch_pdl(decode_combine_kernel<256>, grid, block, 0, s, p);
+    case 64: return launch_pdl(decode_combine_kernel<64, 1>, dim3(pairs), block, 0, s, p);
+    case 128:
+      return split ? launch_pdl(decode_combine_kernel<128, 2>, dim3(pairs * 2), block, 0, s, p)
+                   : launch_pdl(decode_combine_kernel<128, 1>, dim3(pairs), block, 0, s, p);
+    case 256:
+      return split ? launch_pdl(decode_combine_kernel<256, 4>, dim3(pairs * 4), block, 0, s, p)
+                   : launch_pdl(decode_combine_kernel<256, 1>, dim3(pairs), block, 0, s, p);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -180,7 +180,7 @@ cudaError_t launch_decode(const DecodeParams& p, const CUtensorMap& k_map,
                           const CUtensorMap& v_map, int head_dim, int grid, cudaStream_t s,
                           bool fp8 = false);
 cudaError_t launch_calib_combine(const CalibCombineParams& p, int head_dim, cudaStream_t s);
-cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, cudaStream_t s);
+cudaError_t launch_decode_combine(const DecodeParams& p, int head_dim, int num_sms, cudaStream_t s);
 // fp8: q and the K/V tiles are staged 8-bit-cache rows in fp16 (fp16 mmas)
 cudaError_t launch_prefill_tc(const PrefillParams& p, int head_dim, const CUtensorMap& q_map,
                               const CUtensorMap& ck_map, const CUtensorMap& cv_map,

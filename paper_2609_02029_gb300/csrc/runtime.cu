@@ -643,7 +643,7 @@ static hwkv_status decode_call(hwkv_cache* c, int32_t layer, const void* q, cons
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   cudaError_t e = launch_decode(p, c->kv_map, c->kv_map, c->pol.head_dim, grid, s, c->fp8());
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
-  e = launch_decode_combine(p, c->pol.head_dim, s);
+  e = launch_decode_combine(p, c->pol.head_dim, c->num_sms, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
   if (mode == kFused)
     for (int b = 0; b < B; ++b)
@@ -924,7 +924,7 @@ hwkv_status hwkv_decode_attn_static(hwkv_cache* c, int32_t layer, const void* q,
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   e = launch_decode(p, c->kv_map, c->kv_map, d, grid, s, c->fp8());
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "decode launch: %s", cudaGetErrorString(e));
-  e = launch_decode_combine(p, d, s);
+  e = launch_decode_combine(p, d, c->num_sms, s);
   if (e != cudaSuccess) return fail(HWKV_ECUDA, "combine launch: %s", cudaGetErrorString(e));
   return ok();
 }
