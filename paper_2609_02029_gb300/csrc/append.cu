@@ -7,8 +7,10 @@
 // own first position t0 (ragged rows). A new token whose window slot a later
 // token of the same call takes is not written (nor read). Block 0 also stores the
 // rows' new lengths in the device length array. One launch covers every KV head
-// and batch row of a layer (grid y and z); each thread moves 16-byte vectors of the
-// rows that land, reads coalesced within each input row and writes over the ring rows.
+// and batch row of a layer: grid z is the batch row, grid x is laid out head by head,
+// each head's range sized for the rows it can keep (min(n, cap)). Each thread moves
+// 16-byte vectors of the rows that land, reads coalesced within each input row and
+// writes over the ring rows.
 #include <algorithm>
 
 #include "hwkv_internal.cuh"
@@ -60,8 +62,9 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
 }
 
 // The 8-bit format (E4M3 codes, one fp32 scale per stored row), laid out as the
-// bf16 kernel: block (x, h, b) takes the landing tokens of KV head h of batch row b;
-// each half warp quantizes one token row (K and V), each lane D/16 consecutive
+// bf16 kernel: the blocks of head h's range in grid x and row b in grid z take the
+// landing tokens of KV head h of batch row b; each half warp quantizes one token row
+// (K and V), each lane D/16 consecutive
 // channels (a half-warp row needs one shuffle step less per value than a warp row
 // and spreads each row's index arithmetic over twice the values).
 // amax = max |x|; s = the smallest power of two >= amax / 448; code = E4M3 of x / s
