@@ -435,6 +435,7 @@ def run_secondary(args, name, world, rank, local, hbm):
     a = argparse.Namespace(**vars(args))
     a.steps, a.e2e_steps = min(args.steps, 32), min(args.e2e_steps, 8)
     r = run_gpu(a, wl, world, rank, local)
+    graph_gbs = r["step_bytes"] / (r["graph_ms"] / r["graph_steps"] * 1e-3) / 1e9
     return {"workload": wl.name, "layers": wl.n_layers, "batch_per_gpu": wl.batch,
             "head_dim": wl.head_dim, "context": wl.max_ctx, "windows": wl.note,
             "value": r["value"], "unit": "tokens/s", "steps": a.steps,
@@ -444,7 +445,10 @@ def run_secondary(args, name, world, rank, local, hbm):
             "decode_gbs": r["achieved_gbs"], "frac": r["achieved_gbs"] / hbm,
             "bytes_per_launch": r["bytes_avg"], "launch_ms": r["dec_avg_ms"],
             "step_bytes": r["step_bytes"],
-            "graph_step_gbs": r["step_bytes"] / (r["graph_ms"] / r["graph_steps"] * 1e-3) / 1e9,
+            "graph_step_gbs": graph_gbs,
+            # the whole replayed step (every layer's split and combine launches) against
+            # the copy bandwidth; frac above is one eager layer launch
+            "graph_frac": graph_gbs / hbm,
             "l2": ("each timed step preceded by a 2 x L2 read outside its events"
                    if r["flush"] else "inputs larger than L2"),
             "residency_bytes": r["resid_bytes"]}
