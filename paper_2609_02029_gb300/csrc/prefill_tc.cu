@@ -74,7 +74,11 @@ struct TcCfg {
   // a softmax warp may run a key tile ahead of the PV issuer, so a per-tile barrier
   // could complete two phases before it is waited on), else one per query tile
   static constexpr int kPBars = PS ? QT * SBUF : QT;
-  static constexpr int kNumBars = 2 * KST + 2 * VST + 2 * QT * SBUF + 2 * kPBars + 4;
+  // With P over 128-key S tiles the softmax writes P in two 64-key chunks, the chunk it
+  // still holds in registers first; a barrier on that half lets the PV product over
+  // its 64 keys start while the softmax works on the other chunk
+  static constexpr bool kHalfP = PS && BN == 128;
+  static constexpr int kNumBars = 2 * KST + 2 * VST + 2 * QT * SBUF + 3 * kPBars + 4;
   static constexpr int kBarBytes = 512;
   static_assert(8 * kNumBars + 4 <= kBarBytes, "barriers and the TMEM address slot");
   // the dynamic shared memory window starts 1024-aligned (the kernel checks it)
@@ -254,7 +258,8 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
   uint64_t* q_full = pv_done + C::kPBars;
   uint64_t* o_full = q_full + 1;
   uint64_t* drain = o_full + 1;               // [2] each issuer's mmas done
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
+  uint64_t* p_half = drain + 2;               // [kPBars] first P chunk written (kHalfP)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(p_half + C::kPBars);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = p.group;
@@ -286,6 +291,7 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
     }
     for (int i = 0; i < C::kPBars; ++i) {
       mbar_init(&p_full[i], 4);  // one arrival per warp of the tile's warpgroup
+      mbar_init(&p_half[i], 4);
       mbar_init(&pv_done[i], 1);
     }
     mbar_init(q_full, 1);
@@ -494,17 +500,27 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
         const uint32_t v_base = smem_u32(sV + (j % VST) * C::kTileBytes);
 #pragma unroll
         for (int t = 0; t < QT; ++t) {
-          ok = ok && wait_or_abort(&p_full[C::p_bar(t, j)], C::p_parity(j), p.err, aborted);
-          if (ok) {
+          // 16 keys = 8 packed P columns; with kHalfP keys 64 .. 127 (the chunk the
+          // softmax writes first) go as soon as their P is written, then keys 0 .. 63
+          auto pv_keys = [&](int kk0, int kk1, bool first) {
             tc_fence_after();
 #pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk) {  // 16 keys = 8 packed P columns
+            for (int kk = kk0; kk < kk1; ++kk) {
               const uint64_t bd = smem_desc_sw128(v_base + kk * 2048, C::kKVSlab, 1024);
               umma_bf16_tmem_a(tmem + C::kColO + t * D, tmem + C::col_p(t, j) + C::p_chunk_col(kk / 4) + (kk % 4) * 8, bd,
-                               idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+                               idesc_pv, (j > 0 || !first || kk > kk0) ? 1u : 0u);
             }
-            umma_commit(&pv_done[C::p_bar(t, j)]);
+          };
+          if constexpr (C::kHalfP) {
+            ok = ok && wait_or_abort(&p_half[C::p_bar(t, j)], C::p_parity(j), p.err, aborted);
+            if (ok) pv_keys(4, 8, true);
+            ok = ok && wait_or_abort(&p_full[C::p_bar(t, j)], C::p_parity(j), p.err, aborted);
+            if (ok) pv_keys(0, 4, false);
+          } else {
+            ok = ok && wait_or_abort(&p_full[C::p_bar(t, j)], C::p_parity(j), p.err, aborted);
+            if (ok) pv_keys(0, BN / 16, true);
           }
+          if (ok) umma_commit(&pv_done[C::p_bar(t, j)]);
         }
         if (ok) umma_commit(&v_empty[j % VST]);  // every query tile's PV has read it
         ++j;
@@ -666,6 +682,14 @@ __global__ void __launch_bounds__(TcCfg<D, BN, KST, VST, QT, SBUF, CTAS, PS, F16
           rescale_o();
         }
         tmem_st32(t_lane + C::col_p(tq, j) + C::p_chunk_col(ch), *reinterpret_cast<const uint32_t(*)[32]>(&sv[0]));
+        if constexpr (C::kHalfP) {
+          if (cc == 0) {  // this chunk's P (and any O rescale before it) is in TMEM
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_half[C::p_bar(tq, j)]);
+          }
+        }
       }
       tmem_st_wait();
       float s4[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
