@@ -45,7 +45,7 @@ DECODE_TRAFFIC_PER_BYTE = (244.291584e6 + 4.332032e6) / 244064256.0
 # tensor-pipe activity of the prefill kernel (ncu sm__pipe_tensor_cycles_active, pct of peak
 # sustained active) from the one-launch --set full capture summarised in the named profile;
 # set to None whenever that kernel changes.
-PREFILL_TENSOR_PIPE = {"prefill64k": (0.507, "profiles/prefill_tc_prefill64k_full.md")}
+PREFILL_TENSOR_PIPE = {"prefill64k": (0.512, "profiles/prefill_tc_prefill64k_full.md")}
 
 
 def peaks():
