@@ -15,8 +15,7 @@ import pytest
 import hwkv_gen
 import oracle
 import paper_2609_02029_gb300 as hwkv
-from harness import Run
-from test_gpu_sink import RunS
+from harness import Run, RunS
 
 pytestmark = pytest.mark.gpu
 BF16, FP8 = hwkv.HWKV_KV_BF16, hwkv.HWKV_KV_FP8_E4M3
