@@ -696,12 +696,13 @@ __global__ void __launch_bounds__((kDecodeWarps + 1) * 32, 1)
 // o = sum_j 2^{(m_j - M) c} o_j / sum_j 2^{(m_j - M) c} l_j, M = max_j m_j.
 // CH CTAs of 8 warps per (batch row, query head), each over D / CH consecutive
 // channels (CH > 1 for small steps, with few (batch row, query head) pairs: the merge
-// is spread over more SMs and each warp takes more partials per round). Warp w merges partials w, w + 8, w + 16, ... in that order with a running
-// maximum (each lane D / (32 CH) consecutive channels), loading a batch of partials
-// (32 floats per lane) before using any of them, so a ring split over many CTAs costs
-// a few rounds of L2 latency rather than one per partial; the eight warps' results
-// are then merged in warp order (deterministic). Rings read whole by one CTA were
-// written by the split kernel.
+// is spread over more SMs and each warp takes more partials per round). Warp w merges
+// partials w, w + 8, w + 16, ... in that order with a running maximum (each lane
+// D / (32 CH) consecutive channels), loading a batch of partials (32 floats per lane)
+// before using any of them, so a ring split over many CTAs costs a few rounds of L2
+// latency rather than one per partial; the eight warps' results are then merged in
+// warp order (deterministic). Rings read whole by one CTA were written by the split
+// kernel.
 constexpr int kCombineWarps = 8;
 
 template <int D, int CH>
