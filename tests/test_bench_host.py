@@ -104,3 +104,25 @@ def test_oracle_layer_steps_cover_every_unit():
     assert keys == wl.batch * sum(p - oracle.window_lo(p, 0 if W >= wl.max_ctx else W) + 1
                                   for W in wl.windows)
     assert sec > 0
+
+
+def test_secondary_line_rates():
+    """The secondary workload line divides each step's bytes by the replayed graph's
+    step time and reports it against the copy bandwidth (graph_frac) beside the one
+    eager layer launch (frac); the GPU run is replaced by fixed timings."""
+    import argparse
+    fake = {"value": 100.0, "ms": 80.0, "graph_value": 110.0, "graph_ms": 40.0, "graph_steps": 8,
+            "e2e_value": 90.0, "achieved_gbs": 5000.0, "bytes_avg": 1.0e9, "dec_avg_ms": 0.2,
+            "step_bytes": 3.0e9, "flush": False, "resid_bytes": 123}
+    saved = bench.run_gpu
+    bench.run_gpu = lambda a, wl, world, rank, local: fake
+    try:
+        args = argparse.Namespace(steps=96, e2e_steps=32)
+        line = bench.run_secondary(args, "budget161k_r25", 1, 0, 0, 6000.0)
+    finally:
+        bench.run_gpu = saved
+    assert line["steps"] == 32
+    assert line["graph_ms_per_step"] == 40.0 / 8
+    assert abs(line["graph_step_gbs"] - 3.0e9 / (5.0e-3) / 1e9) < 1e-9
+    assert abs(line["graph_frac"] - line["graph_step_gbs"] / 6000.0) < 1e-12
+    assert abs(line["frac"] - 5000.0 / 6000.0) < 1e-12
